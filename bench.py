@@ -1,0 +1,403 @@
+"""Throughput of the RelaySum step (RelaySGD, arXiv 2110.04175, Algorithm 1).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
+                    [--workload NAME] [--e2e-steps K2] [--no-cpu-baseline]
+
+A step is one RelaySGD iteration of the whole hot path -- counter update,
+local step with Philox gradient noise, every relay message, every rebuild --
+over the default workload: 32 workers on a balanced binary tree, d = 1.1e8
+fp32 parameters each (a BERT-base-sized flat vector), robust rebuild.  The
+per-step working set (82.7 GB moved) is far larger than L2, so no flush is
+needed between steps.  Inputs are seeded synthetic quadratics.
+
+Prints one JSON line.  `value` is whole-job steps/s with the state resident
+in HBM; `e2e` is the same metric through relay_step with the state in pinned
+host buffers (copies inside the timed region); `roofline` is the fused
+kernel's algorithmic HBM bytes per launch over its CUDA-event duration;
+`cpu_baseline` times the plain CPU oracle on a bounded coordinate sample.
+
+Multi-GPU (torchrun, one rank per GPU): every rank runs the same workload on
+its own d-slice of one longer model vector (coordinates are independent, so
+there is no data-path collective; weak scaling).  `--impl reference` times
+the CPU oracle instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "RelaySum steps/s and achieved HBM GB/s (fraction of GB300 peak) vs CPU oracle"
+DEFAULT_WORKLOAD = "binary32_d110000000"
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ------------------------------------------------------------ host helpers
+
+def shard_offset(rank: int, d: int) -> int:
+    """First absolute coordinate of rank `rank`'s slice (multiple of 4)."""
+    return rank * ((d + 3) // 4 * 4)
+
+
+def reduce_max(value: float, world: int) -> float:
+    """Max over ranks (the slowest rank sets the job time)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def measured_peaks() -> dict:
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return json.load(f)
+    except (OSError, ValueError):
+        return {}
+
+
+class ClockSampler:
+    """nvidia-smi samples (every 200 ms) of the GPU's clocks and throttle
+    reasons while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, bus_id: str | None):
+        self.proc = None
+        self.file = None
+        self.bus_id = bus_id
+
+    def __enter__(self):
+        try:
+            self.file = tempfile.TemporaryFile(mode="w+")
+            cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                   "-lms", "200"]
+            if self.bus_id:
+                cmd += ["-i", self.bus_id]
+            self.proc = subprocess.Popen(cmd, stdout=self.file, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.file is None:
+            return None
+        self.file.seek(0)
+        rows = [r.split(",") for r in self.file.read().strip().splitlines() if r.strip()]
+        samples = []
+        for r in rows:
+            try:
+                samples.append({"sm": float(r[1]), "max": float(r[2]), "power": float(r[3]),
+                                "hw": r[5].strip(), "hw_thermal": r[6].strip(),
+                                "sw_thermal": r[7].strip(), "sw_power": r[8].strip()})
+            except (ValueError, IndexError):
+                continue
+        if not samples:
+            return None
+        peak_power = max(s["power"] for s in samples)
+        loaded = [s for s in samples if s["power"] >= 0.5 * peak_power] or samples
+        reasons = set()
+        for s in loaded:
+            for key, name in (("hw", "hw_slowdown"), ("hw_thermal", "hw_thermal_slowdown"),
+                              ("sw_thermal", "sw_thermal_slowdown"), ("sw_power", "sw_power_cap")):
+                if s[key].lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(s["sm"] for s in loaded),
+                "sm_max_mhz": max(s["max"] for s in samples),
+                "reasons": sorted(reasons), "samples": len(samples), "samples_under_load": len(loaded),
+                "power_w_max": peak_power}
+
+
+def bus_id_of(device: int) -> str | None:
+    """nvidia-smi's id (its PCI bus id) of the torch device, or None."""
+    import torch
+    p = torch.cuda.get_device_properties(device)
+    want = tuple(getattr(p, k, None) for k in ("pci_domain_id", "pci_bus_id", "pci_device_id"))
+    try:
+        out = subprocess.run(["nvidia-smi", "--query-gpu=pci.bus_id", "--format=csv,noheader"],
+                             capture_output=True, text=True, timeout=30).stdout
+    except (OSError, subprocess.SubprocessError):
+        return None
+    ids = [line.strip() for line in out.splitlines() if line.strip()]
+    for bus in ids:
+        try:
+            dom, b, rest = bus.split(":")
+            if (int(dom, 16), int(b, 16), int(rest.split(".")[0], 16)) == want:
+                return bus
+        except ValueError:
+            continue
+    return ids[0] if len(ids) == 1 else None
+
+
+# -------------------------------------------------------------- CPU oracle
+
+def oracle_sample(w, seconds: float = 15.0, max_len: int = 1 << 20):
+    """Times the oracle (as it stands, one thread) on a coordinate slice of
+    workload `w`, scaled to steps/s of the full d."""
+    import numpy as np
+    from oracle import oracle
+    length = 2048
+    st = oracle.State(w.n, w.edges, length)
+    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+    t0 = time.perf_counter()
+    st.advance(1, w.lr, w.sigma, w.seed, w.mode)
+    per_coord_step = (time.perf_counter() - t0) / length
+    steps = 4
+    length = int(min(max_len, w.d, max(1024, seconds / (steps * per_coord_step))))
+    st = oracle.State(w.n, w.edges, length)
+    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+    t0 = time.perf_counter()
+    st.advance(steps, w.lr, w.sigma, w.seed, w.mode)
+    dt = time.perf_counter() - t0
+    return {"value": steps / dt * length / w.d, "unit": "steps/s", "cores": 1, "kind": "oracle",
+            "sample": f"{steps} steps of coordinates [0, {length}) of d = {w.d} "
+                      f"({dt:.1f} s, one thread), scaled by {length}/{w.d}"}
+
+
+def run_reference(args, w, rank: int):
+    """The reference arm: the plain CPU oracle on bounded samples of the
+    same workload; each step is one oracle step over a coordinate slice."""
+    import numpy as np
+    from oracle import oracle
+    if rank != 0:
+        return
+    length = 4096
+    st = oracle.State(w.n, w.edges, length)
+    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+    t0 = time.perf_counter()
+    st.advance(1, w.lr, w.sigma, w.seed, w.mode)
+    per_coord = (time.perf_counter() - t0) / length
+    budget = 90.0 / max(1, args.steps + args.warmup)
+    length = int(max(256, min(1 << 20, w.d, budget / per_coord)))
+    st = oracle.State(w.n, w.edges, length)
+    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+    st.advance(args.warmup, w.lr, w.sigma, w.seed, w.mode)
+    t0 = time.perf_counter()
+    st.advance(args.steps, w.lr, w.sigma, w.seed, w.mode)
+    dt = time.perf_counter() - t0
+    value = args.steps / dt * length / w.d
+    sample = (f"each step: one oracle step over coordinates [0, {length}) of d = {w.d}, "
+              f"one thread; steps/s scaled by {length}/{w.d}")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dt / args.steps * 1e3 * w.d / length, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(w, args.gpus),
+            "cpu_baseline": {"value": value, "unit": "steps/s", "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(w, gpus: int) -> dict:
+    shape = {"binary": "balanced binary tree (heap order)", "chain": "chain", "star": "star",
+             "torus": "uniform spanning tree of the 8x8 torus"}
+    kind = next((v for k, v in shape.items() if w.name.startswith(k)), w.name)
+    return {"workload": w.name, "n_workers": w.n, "tree": kind, "d": w.d, "directed_edges": w.E,
+            "rebuild": "robust (Section 4.4)" if w.mode == 1 else "Algorithm 1",
+            "sigma": w.sigma, "lr": w.lr, "objective": "identity-Hessian heterogeneous quadratics",
+            "l2": f"inputs larger than L2 ({w.bytes_per_step() / 1e9:.1f} GB moved per step)",
+            "parallelism": f"d-sharded over {gpus} rank(s), no collective" if gpus > 1
+            else "1 GPU"}
+
+
+# ------------------------------------------------------------------ native
+
+def run_native(args, w, rank: int, world: int):
+    import numpy as np
+    import torch
+
+    import paper_2110_04175_gb300 as rs
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    c0 = shard_offset(rank, w.d)
+    run = rs.RelayRun(w.n, w.d, w.edges, device=dev, mode=w.mode, c0=c0)
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    h = run.h
+
+    def one_step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        rs.relay_step_counts(h, run.counts, stream)
+        if ev is not None:
+            ev[1].record(stream)
+        rs.relay_step_models(h, run.x, run.msg[run.cur], run.msg[1 - run.cur], run.counts, w.lr,
+                             w.seed, run.t, stream)
+        if ev is not None:
+            ev[2].record(stream)
+        run.cur = 1 - run.cur
+        run.t += 1
+
+    for _ in range(args.warmup):
+        one_step()
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    with ClockSampler(bus_id_of(local) if rank == 0 else None) as clocks:
+        for k in range(args.steps):
+            one_step(events[k])
+        torch.cuda.synchronize(dev)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    total_ms = events[0][0].elapsed_time(events[-1][2])
+    models_ms = [events[k][1].elapsed_time(events[k][2]) for k in range(args.steps)]
+    total_ms = reduce_max(total_ms, world)
+    steps_per_s = world * args.steps / (total_ms / 1e3)
+
+    # end to end: state in pinned host memory, copied in and out every step
+    e2e = None
+    if args.e2e_steps > 0:
+        e2e = run_e2e(args, w, run, dev, stream, world)
+
+    if rank != 0:
+        return
+    peaks = measured_peaks()
+    peak = peaks.get("hbm_gbs")
+    peak_src = "measured" if peak else "fallback"
+    peak = peak or FALLBACK_HBM_GBS
+    mean_models_ms = statistics.mean(models_ms)
+    alg_bytes = w.bytes_per_step()
+    achieved = alg_bytes / (mean_models_ms / 1e3) / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": traffic_per_launch(w),
+                "kernel": "relay_models_kernel", "peak_source": peak_src,
+                "algorithmic_bytes_per_launch": alg_bytes,
+                "bytes_per_launch_incl_mu": w.bytes_per_step_with_mu(),
+                "achieved_incl_mu": round(w.bytes_per_step_with_mu() / (mean_models_ms / 1e3) / 1e9,
+                                          1),
+                "launch_ms_mean": round(mean_models_ms, 4),
+                "launch_ms_min": round(min(models_ms), 4)}
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        cpu = oracle_sample(w)
+    line = {"metric": METRIC, "value": round(steps_per_s, 4), "unit": "steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": workload_config(w, world), "roofline": roofline, "cpu_baseline": cpu,
+            "e2e": e2e, "gpu_launches": 2 * args.steps, "clocks": clocks.summary(),
+            "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1)}
+    print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, w, run, dev, stream, world: int):
+    """relay_step with x, messages and counters living in pinned host memory:
+    every step copies them to the device, runs, and copies the results back."""
+    import torch
+
+    import paper_2110_04175_gb300 as rs
+
+    hx = torch.empty_like(run.x, device="cpu").pin_memory()
+    hm_in = torch.empty_like(run.msg[0], device="cpu").pin_memory()
+    hm_out = torch.empty_like(run.msg[0], device="cpu").pin_memory()
+    hc = torch.empty_like(run.counts, device="cpu").pin_memory()
+    hx.copy_(run.x)
+    hm_in.copy_(run.msg[run.cur])
+    hc.copy_(run.counts)
+    torch.cuda.synchronize(dev)
+    h2d = (hx.numel() + hm_in.numel() + hc.numel()) * 4
+    d2h = (hx.numel() + hm_out.numel() + hc.numel()) * 4
+    barrier(world)
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(args.e2e_steps):
+        run.x.copy_(hx, non_blocking=True)
+        run.msg[0].copy_(hm_in, non_blocking=True)
+        run.counts.copy_(hc, non_blocking=True)
+        rs.relay_step(run.h, run.x, run.msg[0], run.msg[1], run.counts, w.lr, w.seed, run.t, stream)
+        hx.copy_(run.x, non_blocking=True)
+        hm_out.copy_(run.msg[1], non_blocking=True)
+        hc.copy_(run.counts, non_blocking=True)
+        run.t += 1
+        hm_in, hm_out = hm_out, hm_in
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = reduce_max(start.elapsed_time(end), world)
+    return {"value": round(world * args.e2e_steps / (ms / 1e3), 4), "unit": "steps/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
+            "path": "relay_step with x, messages and counters in pinned host memory"}
+
+
+def traffic_per_launch(w):
+    """DRAM bytes per launch of the fused kernel from the committed ncu
+    summary for this workload, if one exists (None otherwise)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            return json.load(f).get(w.name)
+    except (OSError, ValueError):
+        return None
+
+
+def main(argv=None):
+    p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawTextHelpFormatter)
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=50)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["native", "reference"], default="native")
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    args = p.parse_args(argv)
+    if args.warmup < 3:
+        p.error("--warmup must be >= 3")
+
+    from paper_2110_04175_gb300 import workloads as wl
+    w = wl.by_name(args.workload)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, w, rank)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        dist.init_process_group("nccl")
+    try:
+        run_native(args, w, rank, world)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,159 @@
+/*
+ * relaysum.h -- C ABI of the GB300 RelaySum step library (librelaysum.so).
+ *
+ * One RelaySGD iteration (Vogels et al., "RelaySum for Decentralized Deep
+ * Learning on Heterogeneous Data", arXiv 2110.04175, Algorithm 1) for n
+ * virtual workers of a spanning tree, all resident on one GPU:
+ *
+ *   local step     x_i^{t+1/2} = x_i^t - lr * ((x_i^t - mu_i) + sigma * xi_i^t)
+ *   relay message  m_{i->j}^t  = x_i^{t+1/2} + sum_{k in N(i)\j} m_{k->i}^{t-1}
+ *   counter        c_{i->j}^t  = 1 + sum_{k in N(i)\j} c_{k->i}^{t-1}
+ *   models seen    nbar_i      = 1 + sum_{j in N(i)} c_{j->i}^t
+ *   rebuild        mode 0 (Alg. 1):  x_i^{t+1} = (x_i^{t+1/2} + sum_j m_{j->i}^t) / nbar_i
+ *                  mode 1 (robust rule of Section 4.4):
+ *                      x_i^{t+1} = (x_i^{t+1/2} + sum_j m_{j->i}^t + (n - nbar_i) x_i^t) / n
+ *
+ * The objective is the synthetic heterogeneous quadratic f_i = 1/2||x - mu_i||^2
+ * with Philox4x32-10 gradient noise xi (the appendix "Independence of
+ * heterogeneity" adds random normal noise to each gradient update).
+ *
+ * Conventions shared by every call:
+ *   - Layout.  x and mu are fp32 [n][ld], messages fp32 [E][ld] with
+ *     E = 2(n-1), counters int32 [E]; ld = relay_ld(h) >= d is the padded
+ *     row stride (a multiple of 32 floats).  Columns [d, ld) are padding:
+ *     the library zeroes them on init and never reads them as data.
+ *     Undirected edge u of the edge list gives directed edges 2u
+ *     (edges[2u] -> edges[2u+1]) and 2u+1 (the reverse).
+ *   - Ownership.  The caller allocates and owns every device buffer; a
+ *     handle owns only its host-side tables.  No call allocates device
+ *     memory, and no call synchronises: device work is enqueued on `stream`
+ *     (a cudaStream_t; NULL is the legacy default stream) of the current
+ *     device.
+ *   - Errors.  Every int-returning call returns RELAY_OK (0) or a negative
+ *     status; arguments are checked before anything is enqueued, and a
+ *     rejected call leaves every buffer untouched.  RELAY_ECUDA reports a
+ *     failed launch (cudaGetLastError); no C++ exception crosses the ABI.
+ *   - Random numbers.  Philox4x32-10 (Salmon et al., SC'11) with key
+ *     (seed lo32, seed hi32) and counter (q, row, step, stream) where q is
+ *     the ABSOLUTE coordinate quad (c0 + c) / 4; stream 0 = gradient noise
+ *     of worker `row` at `step`, 1 = Gaussian centre `row`, 2 = the shared
+ *     initial model.  Words (0,1) and (2,3) become two Box-Muller pairs
+ *     for coordinates 4q, 4q+1 and 4q+2, 4q+3, via u = ((w >> 8) + 1) 2^-24.
+ */
+#ifndef RELAYSUM_H
+#define RELAYSUM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define RELAY_OK 0
+#define RELAY_EINVAL (-1)        /* bad argument (null pointer, range, aliasing) */
+#define RELAY_ENOTTREE (-2)      /* the edge list is not a tree on 0..n-1        */
+#define RELAY_ECUDA (-3)         /* a CUDA launch or runtime call failed         */
+#define RELAY_ENOMEM (-4)        /* host allocation failed                       */
+#define RELAY_EUNSUPPORTED (-5)  /* n > RELAY_MAX_N, or a size beyond the limits */
+
+#define RELAY_MAX_N 256          /* workers per handle                            */
+
+typedef struct relay_handle relay_handle;
+typedef struct CUstream_st *relay_stream_t; /* identical to cudaStream_t */
+
+/* Creates a handle for n >= 1 workers with d >= 0 parameters each on the
+ * tree given by n_edges = n - 1 undirected pairs `edges` (host, int32
+ * [n_edges][2], ids in 0..n-1).  Validates that the pairs form a tree
+ * (Section 3 "Setup": no self loops; Alg. 1 runs on a tree) and builds the
+ * per-node visit program of the fused kernel.  Host work only: no CUDA call.
+ * Errors: RELAY_EINVAL (out == NULL, d < 0, d with (d+31)/4 >= 2^32 quads),
+ * RELAY_ENOTTREE, RELAY_EUNSUPPORTED (n > RELAY_MAX_N), RELAY_ENOMEM. */
+int relay_create(relay_handle **out, int32_t n, int64_t d, const int32_t *edges,
+                 int32_t n_edges);
+
+/* Releases a handle (NULL is allowed).  Device buffers are the caller's. */
+void relay_destroy(relay_handle *h);
+
+/* Padded row stride in floats: d rounded up to a multiple of 32. */
+int64_t relay_ld(const relay_handle *h);
+
+/* Number of directed edges E = 2(n-1) (rows of a message buffer). */
+int32_t relay_num_edges(const relay_handle *h);
+
+/* Directed edge table: src[e] -> dst[e] for e < E (host int32 [E] each).
+ * Edge 2u is edges[u][0] -> edges[u][1], edge 2u+1 its reverse. */
+int relay_edges(const relay_handle *h, int32_t *src, int32_t *dst);
+
+/* Rebuild rule: 0 = Algorithm 1 (divide by nbar), 1 = robust rule of
+ * Section 4.4 (fill the n - nbar missing models with x_i^t, divide by n).
+ * The default is 1. */
+int relay_set_rebuild_mode(relay_handle *h, int32_t mode);
+
+/* Absolute index of this handle's first coordinate within a longer model
+ * vector (c0 >= 0, a multiple of 4): the noise of local coordinate c is
+ * that of coordinate c0 + c, so a vector split into slices -- across GPUs,
+ * or for spot checks -- reproduces the unsplit run exactly.  Default 0. */
+int relay_set_coord_offset(relay_handle *h, int64_t c0);
+
+/* Binds the objective used by every later step: mu is a caller-owned device
+ * fp32 [n][ld] array of quadratic centres (read, never written; it must stay
+ * valid while steps using it run), sigma >= 0 the gradient-noise std. */
+int relay_set_objective(relay_handle *h, const float *mu, float sigma);
+
+/* Fills mu (device fp32 [n][ld]) with mu_i(c) = mu_scale * sum_k
+ * mix[i][k] N_k(c): K Gaussian centres N_k (Philox stream 1, row k) mixed by
+ * the device fp32 [n][K] matrix `mix` (identity for one centre per worker,
+ * Dirichlet rows for a mixture).  Padding columns are set to 0. */
+int relay_fill_objective(relay_handle *h, float *mu, const float *mix, int32_t K,
+                         float mu_scale, uint64_t mu_seed, relay_stream_t stream);
+
+/* Initial state of Algorithm 1: x_i^0 = x0_std * N(c) for every worker (one
+ * shared draw, Philox stream 2), m^{-1} = 0 in msg_a (and in msg_b unless it
+ * is NULL), c^{-1} = 0.  x: device [n][ld]; msg_a, msg_b: device [E][ld];
+ * counts: device int32 [E].  Padding columns are set to 0. */
+int relay_init(relay_handle *h, float *x, float *msg_a, float *msg_b, int32_t *counts,
+               float x0_std, uint64_t seed, relay_stream_t stream);
+
+/* Counter update of Alg. 1 in place: counts c^{t-1} -> c^t (int32 [E]).
+ * Integer, bit-exact.  One 1-CTA launch. */
+int relay_step_counts(relay_handle *h, int32_t *counts, relay_stream_t stream);
+
+/* The per-coordinate part of iteration t in one fused pass over d: local
+ * step, every outgoing relay message and the rebuild, for all workers.
+ * counts must already hold c^t (relay_step_counts ran first); they give
+ * nbar.  x: device [n][ld] in/out (x^t -> x^{t+1}); msg_in: [E][ld] m^{t-1}
+ * (read only); msg_out: [E][ld] m^t (written); msg_in != msg_out, and
+ * neither may overlap x.  lr finite; step in [0, 2^32) is the noise
+ * counter.  RELAY_EINVAL also when no objective is bound. */
+int relay_step_models(relay_handle *h, float *x, const float *msg_in, float *msg_out,
+                       const int32_t *counts, float lr, uint64_t seed, int64_t step,
+                       relay_stream_t stream);
+
+/* One full RelaySGD iteration t: relay_step_counts, then
+ * relay_step_models, enqueued back to back on `stream`.  The caller swaps
+ * msg_in and msg_out before the next step (double-buffered messages). */
+int relay_step(relay_handle *h, float *x, const float *msg_in, float *msg_out,
+               int32_t *counts, float lr, uint64_t seed, int64_t step,
+               relay_stream_t stream);
+
+/* nbar_i = 1 + sum of the counters arriving at i, from host counters
+ * (int32 [E]) into nbar_host (int32 [n]).  Host arithmetic only. */
+int relay_nbar(const relay_handle *h, const int32_t *counts_host, int32_t *nbar_host);
+
+/* Introspection of the fused kernel's visit program (for tests and tools):
+ * number of shared-memory accumulator slots per thread, the visit order
+ * (int32 [n]), per node 8 ints {deg, pos_base, parent_pos, recv_slot,
+ * acc_slot, parent_acc, fin_parent, parent} (int32 [n][8]) and per
+ * position 3 ints {in_edge, out_edge, slot} (int32 [E][3]); any output
+ * pointer may be NULL. */
+int relay_program(const relay_handle *h, int32_t *nslots, int32_t *order, int32_t *node_rec,
+                  int32_t *pos_rec);
+
+/* Static description of a status code. */
+const char *relay_error_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RELAYSUM_H */

@@ -1,0 +1,30 @@
+"""GB300-native RelaySum step (RelaySGD, arXiv 2110.04175, Algorithm 1).
+
+A thin Python binding over the C ABI of ``librelaysum.so`` (declared in
+``include/relaysum.h``): the functions here have the C names and only
+marshal arguments -- torch tensors become device pointers, a torch stream
+becomes a ``cudaStream_t`` -- while every step of the method runs in the
+library's CUDA kernels.  There is no CPU fallback: if the library has not
+been built, the first call raises.
+
+``RelayRun`` is a convenience owner of the device buffers of one run
+(allocated with torch) that swaps the double-buffered messages between
+steps.
+"""
+from __future__ import annotations
+
+from ._native import (RELAY_EINVAL, RELAY_ECUDA, RELAY_ENOMEM, RELAY_ENOTTREE, RELAY_EUNSUPPORTED,
+                      RELAY_MAX_N, RELAY_OK, RelayError, RelayHandle, RelayRun, library_path,
+                      relay_create, relay_destroy, relay_edges, relay_error_string,
+                      relay_fill_objective, relay_init, relay_ld, relay_nbar, relay_num_edges,
+                      relay_program, relay_set_coord_offset, relay_set_objective,
+                      relay_set_rebuild_mode, relay_step, relay_step_counts, relay_step_models)
+
+__all__ = [
+    "RELAY_OK", "RELAY_EINVAL", "RELAY_ENOTTREE", "RELAY_ECUDA", "RELAY_ENOMEM",
+    "RELAY_EUNSUPPORTED", "RELAY_MAX_N", "RelayError", "RelayHandle", "RelayRun", "library_path",
+    "relay_create", "relay_destroy", "relay_ld", "relay_num_edges", "relay_edges",
+    "relay_set_rebuild_mode", "relay_set_coord_offset", "relay_set_objective",
+    "relay_fill_objective", "relay_init", "relay_step_counts", "relay_step_models", "relay_step",
+    "relay_nbar", "relay_program", "relay_error_string",
+]

@@ -1,0 +1,599 @@
+// relaysum.cu -- GB300 (sm_103a) kernels and C ABI of the RelaySum step.
+//
+// Vogels et al., "RelaySum for Decentralized Deep Learning on Heterogeneous
+// Data" (arXiv 2110.04175), Algorithm 1 (RelaySGD) with the robust rebuild of
+// Section 4.4, for n virtual workers on one GPU.  See relaysum.h for the
+// equations and the ABI contract, program.h for the visit program.
+//
+// Kernels:
+//   relay_counts_kernel   Alg. 1 counters, int32, one CTA, in place.
+//   relay_models_kernel   everything per coordinate, in ONE pass over d:
+//                         local step with Philox noise, every outgoing relay
+//                         message, every rebuild.  Each x_i, mu_i and incoming
+//                         message quad is read from HBM once and each outgoing
+//                         message / new model quad written once (the generic
+//                         path for degree > 4 re-reads its incoming messages
+//                         once more, from cache).  The path is bandwidth-bound
+//                         streaming arithmetic: no tensor cores.
+//   relay_init_kernel     x^0 (shared Philox draw) and zeroed messages.
+//   relay_fill_mu_kernel  mu_i = scale * sum_k mix[i][k] N_k.
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <new>
+
+#include "program.h"
+#include "relaysum.h"
+
+using relaysum::kMaxE;
+using relaysum::kMaxN;
+using relaysum::kRegDeg;
+using relaysum::NodeRec;
+using relaysum::Program;
+
+struct relay_handle {
+    Program prog;
+    int64_t d = 0, ld = 0, nquads = 0, c0 = 0;
+    int32_t mode = 1;
+    const float* mu = nullptr;
+    float sigma = 0.0f;
+    bool has_objective = false;
+};
+
+namespace {
+
+// ------------------------------------------------------------ random numbers
+
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): round multipliers and
+// Weyl key increments of the published definition.
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u;
+constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;
+constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
+
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+    for (int round = 0; round < 10; ++round) {
+        const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
+        const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
+        c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+        k0 += kPhiloxW0;
+        k1 += kPhiloxW1;
+    }
+    return c;
+}
+
+// 24 high bits -> (0, 1], exact in fp32.
+__device__ __forceinline__ float unit_interval(uint32_t w) {
+    return __uint2float_rn((w >> 8) + 1u) * 5.9604644775390625e-8f;  // 2^-24
+}
+
+// Four standard normals for coordinates 4q .. 4q+3 (Box-Muller on the two
+// word pairs of one Philox block).
+__device__ __forceinline__ float4 normal4(uint32_t q, uint32_t row, uint32_t step, uint32_t stream,
+                                          uint32_t k0, uint32_t k1) {
+    const uint4 w = philox4x32_10(make_uint4(q, row, step, stream), k0, k1);
+    const float r0 = sqrtf(-2.0f * logf(unit_interval(w.x)));
+    const float r1 = sqrtf(-2.0f * logf(unit_interval(w.z)));
+    float s0, c0, s1, c1;
+    sincospif(2.0f * unit_interval(w.y), &s0, &c0);
+    sincospif(2.0f * unit_interval(w.w), &s1, &c1);
+    return make_float4(r0 * c0, r0 * s0, r1 * c1, r1 * s1);
+}
+
+// ------------------------------------------------------------ float4 helpers
+
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+    return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+__device__ __forceinline__ float4 scale4(float4 a, float s) {
+    return make_float4(a.x * s, a.y * s, a.z * s, a.w * s);
+}
+__device__ __forceinline__ float4 ld_stream(const float* p) {
+    return __ldg(reinterpret_cast<const float4*>(p));
+}
+__device__ __forceinline__ void st_stream(float* p, float4 v) {
+    __stcs(reinterpret_cast<float4*>(p), v);
+}
+
+// ------------------------------------------------------------------ counters
+
+// c^t_{i->j} = 1 + sum_{k in N(i)\j} c^{t-1}_{k->i}: the incoming edge from
+// j is e ^ 1 for e = i -> j.
+__global__ void relay_counts_kernel(const __grid_constant__ Program prog, int32_t* counts) {
+    __shared__ int32_t c_old[kMaxE];
+    const int E = prog.E;
+    for (int e = threadIdx.x; e < E; e += blockDim.x) c_old[e] = counts[e];
+    __syncthreads();
+    for (int e = threadIdx.x; e < E; e += blockDim.x) {
+        const NodeRec r = prog.node[prog.edge_src[e]];
+        int32_t s = 1;
+        for (int p = 0; p < r.deg; ++p) {
+            const int in = prog.pos_in[r.pos_base + p];
+            if (in != (e ^ 1)) s += c_old[in];
+        }
+        counts[e] = s;
+    }
+}
+
+// --------------------------------------------------------------- fused step
+
+struct ModelArgs {
+    float* x;
+    const float* mu;
+    const float* msg_in;
+    float* msg_out;
+    const int32_t* counts;
+    int64_t ld;       // row stride (floats)
+    int64_t nquads;   // ceil(d / 4)
+    uint32_t q0;      // absolute quad of local coordinate 0
+    uint32_t step;
+    uint32_t k0, k1;  // Philox key
+    float lr, sigma;
+};
+
+// Per-thread view of the shared-memory slots: slot s of this thread is
+// base[s * stride]; a warp's 32 float4 of one slot are contiguous.
+struct Slots {
+    float4* base;
+    int stride;
+    __device__ __forceinline__ float4& operator[](int s) const { return base[s * stride]; }
+};
+
+// The message to the DFS parent joins the parent's accumulator; if this
+// worker is the parent's last child, the parent's rebuild is complete.
+__device__ __forceinline__ void to_parent(const NodeRec& r, const ModelArgs& a, int64_t q, float4 out,
+                                          const Slots& sl, const float* s_scale) {
+    const float4 acc = add4(sl[r.parent_acc], out);
+    if (r.fin_parent >= 0) {
+        st_stream(a.x + r.fin_parent * a.ld + 4 * q, scale4(acc, s_scale[r.fin_parent]));
+    } else {
+        sl[r.parent_acc] = acc;
+    }
+}
+
+// Degree D <= kRegDeg: the D incoming messages live in registers; outgoing
+// message s is prefix(s) + suffix(s+1) with prefix(s) = xh + m_0 + ... + m_{s-1}.
+template <int D>
+__device__ __forceinline__ void visit_small(const Program& prog, const NodeRec& r, const ModelArgs& a,
+                                            int64_t q, float4 xh, const Slots& sl,
+                                            const float* s_scale) {
+    float4 m[D];
+#pragma unroll
+    for (int s = 0; s < D; ++s) m[s] = ld_stream(a.msg_in + prog.pos_in[r.pos_base + s] * a.ld + 4 * q);
+    float4 pre[D];
+    pre[0] = xh;
+#pragma unroll
+    for (int s = 1; s < D; ++s) pre[s] = add4(pre[s - 1], m[s - 1]);
+    float4 suf[D];
+    suf[D - 1] = m[D - 1];
+#pragma unroll
+    for (int s = D - 2; s >= 0; --s) suf[s] = add4(m[s], suf[s + 1]);
+#pragma unroll
+    for (int s = 0; s < D; ++s) {
+        const float4 out = (s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]);
+        st_stream(a.msg_out + prog.pos_out[r.pos_base + s] * a.ld + 4 * q, out);
+        if (s == r.parent_pos) {
+            to_parent(r, a, q, out, sl, s_scale);
+        } else {
+            sl[prog.pos_slot[r.pos_base + s]] = out;
+        }
+    }
+}
+
+// Degree D > kRegDeg: suffix sums go to the node's position slots on a
+// descending pass; an ascending pass re-reads each incoming message (from
+// cache) to extend the prefix and overwrites slot s with message s.
+__device__ __noinline__ void visit_generic(const Program& prog, const NodeRec& r, const ModelArgs& a,
+                                           int64_t q, float4 xh, const Slots& sl,
+                                           const float* s_scale) {
+    const int D = r.deg;
+    const int base = r.pos_base;
+    float4 suf = ld_stream(a.msg_in + prog.pos_in[base + D - 1] * a.ld + 4 * q);
+    sl[prog.pos_slot[base + D - 1]] = suf;
+    for (int s = D - 2; s >= 0; --s) {
+        suf = add4(ld_stream(a.msg_in + prog.pos_in[base + s] * a.ld + 4 * q), suf);
+        sl[prog.pos_slot[base + s]] = suf;
+    }
+    float4 pre = xh;
+    for (int s = 0; s < D; ++s) {
+        const float4 out = (s == D - 1) ? pre : add4(pre, sl[prog.pos_slot[base + s + 1]]);
+        pre = add4(pre, ld_stream(a.msg_in + prog.pos_in[base + s] * a.ld + 4 * q));
+        st_stream(a.msg_out + prog.pos_out[base + s] * a.ld + 4 * q, out);
+        if (s == r.parent_pos) {
+            to_parent(r, a, q, out, sl, s_scale);
+        } else {
+            sl[prog.pos_slot[base + s]] = out;
+        }
+    }
+}
+
+// MODE 0: x' = acc / nbar (Alg. 1).  MODE 1: x' = (acc + (n - nbar) x) / n
+// (robust rule), with the fill term folded into the accumulator up front.
+template <int MODE>
+__global__ void __launch_bounds__(128)
+relay_models_kernel(const __grid_constant__ Program prog, const ModelArgs a) {
+    extern __shared__ float4 slot_mem[];
+    __shared__ float s_scale[kMaxN];
+    __shared__ float s_fill[kMaxN];
+    const int n = prog.n;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const NodeRec r = prog.node[i];
+        int nbar = 1;
+        for (int p = 0; p < r.deg; ++p) nbar += __ldg(a.counts + prog.pos_in[r.pos_base + p]);
+        if (MODE == 0) {
+            s_scale[i] = 1.0f / static_cast<float>(nbar);
+            s_fill[i] = 0.0f;
+        } else {
+            s_scale[i] = 1.0f / static_cast<float>(n);
+            s_fill[i] = static_cast<float>(n - nbar);
+        }
+    }
+    __syncthreads();
+    const Slots sl{slot_mem + threadIdx.x, static_cast<int>(blockDim.x)};
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < a.nquads;
+         q += stride) {
+        for (int v = 0; v < n; ++v) {
+            const int i = prog.order[v];
+            const NodeRec r = prog.node[i];
+            const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld + 4 * q);
+            const float4 mv = ld_stream(a.mu + i * a.ld + 4 * q);
+            const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i),
+                                     a.step, 0u, a.k0, a.k1);
+            // x^{t+1/2} = x - lr * ((x - mu) + sigma * xi)
+            float4 xh;
+            xh.x = fmaf(-a.lr, fmaf(a.sigma, z.x, xv.x - mv.x), xv.x);
+            xh.y = fmaf(-a.lr, fmaf(a.sigma, z.y, xv.y - mv.y), xv.y);
+            xh.z = fmaf(-a.lr, fmaf(a.sigma, z.z, xv.z - mv.z), xv.z);
+            xh.w = fmaf(-a.lr, fmaf(a.sigma, z.w, xv.w - mv.w), xv.w);
+            float4 acc = xh;
+            if (MODE == 1) acc = add4(scale4(xv, s_fill[i]), xh);
+            if (r.recv_slot >= 0) acc = add4(acc, sl[r.recv_slot]);
+            switch (r.deg) {
+                case 0: break;
+                case 1: visit_small<1>(prog, r, a, q, xh, sl, s_scale); break;
+                case 2: visit_small<2>(prog, r, a, q, xh, sl, s_scale); break;
+                case 3: visit_small<3>(prog, r, a, q, xh, sl, s_scale); break;
+                case 4: visit_small<4>(prog, r, a, q, xh, sl, s_scale); break;
+                default: visit_generic(prog, r, a, q, xh, sl, s_scale); break;
+            }
+            if (r.acc_slot < 0) {
+                st_stream(a.x + i * a.ld + 4 * q, scale4(acc, s_scale[i]));
+            } else {
+                sl[r.acc_slot] = acc;
+            }
+        }
+    }
+}
+
+// --------------------------------------------------------------------- init
+
+__global__ void relay_init_kernel(float* x, float* msg_a, float* msg_b, int n, int E, int64_t ld,
+                                  int64_t d, uint32_t q0, float x0_std, uint32_t k0, uint32_t k1) {
+    const int64_t ld4 = ld / 4;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < ld4; q += stride) {
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        const int64_t c = 4 * q;
+        if (c < d) {
+            const float4 z = normal4(q0 + static_cast<uint32_t>(q), 0u, 0u, 2u, k0, k1);
+            v = make_float4(x0_std * z.x, c + 1 < d ? x0_std * z.y : 0.f,
+                            c + 2 < d ? x0_std * z.z : 0.f, c + 3 < d ? x0_std * z.w : 0.f);
+        }
+        for (int i = 0; i < n; ++i) reinterpret_cast<float4*>(x)[i * ld4 + q] = v;
+        const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int e = 0; e < E; ++e) {
+            reinterpret_cast<float4*>(msg_a)[e * ld4 + q] = zero;
+            if (msg_b) reinterpret_cast<float4*>(msg_b)[e * ld4 + q] = zero;
+        }
+    }
+}
+
+__global__ void relay_fill_mu_kernel(float* mu, const float* mix, int n, int K, int64_t ld, int64_t d,
+                                     uint32_t q0, float scale, uint32_t k0, uint32_t k1) {
+    const int64_t ld4 = ld / 4;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < ld4; q += stride) {
+        const int64_t c = 4 * q;
+        for (int i = 0; i < n; ++i) {
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (c < d) {
+                for (int k = 0; k < K; ++k) {
+                    const float w = __ldg(mix + static_cast<int64_t>(i) * K + k);
+                    if (w != 0.0f) {  // a zero weight adds exactly nothing
+                        const float4 z = normal4(q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k),
+                                                 0u, 1u, k0, k1);
+                        acc = make_float4(fmaf(w, z.x, acc.x), fmaf(w, z.y, acc.y),
+                                          fmaf(w, z.z, acc.z), fmaf(w, z.w, acc.w));
+                    }
+                }
+            }
+            const float4 v = make_float4(scale * acc.x, c + 1 < d ? scale * acc.y : 0.f,
+                                         c + 2 < d ? scale * acc.z : 0.f, c + 3 < d ? scale * acc.w : 0.f);
+            reinterpret_cast<float4*>(mu)[i * ld4 + q] = c < d ? v : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    }
+}
+
+// ------------------------------------------------------------- host helpers
+
+constexpr int kMaxDevices = 64;
+// dynamic shared memory cap: 227 KB per CTA minus the static scale/fill tables
+constexpr int kMaxSmem = 224 * 1024;
+
+int device_sms(int* dev_out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+    static std::atomic<int> sms_cache[kMaxDevices];
+    int sms = (dev < kMaxDevices) ? sms_cache[dev].load() : 0;
+    if (sms <= 0) {
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return -1;
+        if (dev < kMaxDevices) sms_cache[dev].store(sms);
+    }
+    *dev_out = dev;
+    return sms;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool overlap(const void* a, int64_t abytes, const void* b, int64_t bbytes) {
+    if (abytes <= 0 || bbytes <= 0) return false;
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(a), b0 = reinterpret_cast<uintptr_t>(b);
+    return a0 < b0 + static_cast<uintptr_t>(bbytes) && b0 < a0 + static_cast<uintptr_t>(abytes);
+}
+
+int launch_status() {
+    return cudaGetLastError() == cudaSuccess ? RELAY_OK : RELAY_ECUDA;
+}
+
+// Threads per CTA for the fused kernel: 128, fewer when the slots would not
+// fit in shared memory.
+int models_threads(int nslots) {
+    int t = 128;
+    while (t > 32 && static_cast<int64_t>(nslots) * t * 16 > kMaxSmem) t -= 32;
+    return t;
+}
+
+template <int MODE>
+int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
+    int dev = 0;
+    const int sms = device_sms(&dev);
+    if (sms <= 0) return RELAY_ECUDA;
+    const int threads = models_threads(h->prog.nslots);
+    const size_t smem = static_cast<size_t>(h->prog.nslots) * threads * 16;
+    if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
+    static std::atomic<bool> smem_set[kMaxDevices];
+    if (smem > 48 * 1024 && dev < kMaxDevices && !smem_set[dev].load()) {
+        if (cudaFuncSetAttribute(relay_models_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kMaxSmem) != cudaSuccess)
+            return RELAY_ECUDA;
+        smem_set[dev].store(true);
+    }
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_models_kernel<MODE>, threads, smem) !=
+            cudaSuccess ||
+        per_sm <= 0)
+        return RELAY_ECUDA;
+    const int64_t want = (a.nquads + threads - 1) / threads;
+    const int64_t cap = static_cast<int64_t>(sms) * per_sm;
+    const int grid = static_cast<int>(want < cap ? want : cap);
+    relay_models_kernel<MODE><<<grid, threads, smem, stream>>>(h->prog, a);
+    return launch_status();
+}
+
+// Argument checks shared by relay_step_models and relay_step.
+int check_step_args(const relay_handle* h, const float* x, const float* msg_in, const float* msg_out,
+                    const int32_t* counts, float lr, int64_t step) {
+    if (!h || !h->has_objective || !std::isfinite(lr)) return RELAY_EINVAL;
+    if (step < 0 || step >= (int64_t(1) << 32)) return RELAY_EINVAL;
+    const int E = h->prog.E;
+    if (E > 0 && !counts) return RELAY_EINVAL;
+    if (h->d == 0) return RELAY_OK;  // counters only
+    if (E > 0 && (!msg_in || !msg_out || msg_in == msg_out)) return RELAY_EINVAL;
+    if (!x || !aligned16(x) || (E > 0 && (!aligned16(msg_in) || !aligned16(msg_out))))
+        return RELAY_EINVAL;
+    const int64_t xb = h->prog.n * h->ld * 4, mb = E * h->ld * 4;
+    if (overlap(x, xb, msg_in, mb) || overlap(x, xb, msg_out, mb) || overlap(msg_in, mb, msg_out, mb))
+        return RELAY_EINVAL;
+    return RELAY_OK;
+}
+
+int grid_for(int64_t items, int threads) {
+    int dev = 0;
+    const int sms = device_sms(&dev);
+    const int64_t want = (items + threads - 1) / threads;
+    const int64_t cap = static_cast<int64_t>(sms > 0 ? sms : 1) * 8;
+    return static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
+}
+
+}  // namespace
+
+// ====================================================================== ABI
+
+extern "C" {
+
+int relay_create(relay_handle** out, int32_t n, int64_t d, const int32_t* edges, int32_t n_edges) {
+    if (out == nullptr) return RELAY_EINVAL;
+    *out = nullptr;
+    if (d < 0) return RELAY_EINVAL;
+    const int64_t ld = (d + 31) / 32 * 32;
+    if (ld / 4 >= (int64_t(1) << 32)) return RELAY_EINVAL;
+    relay_handle* h = new (std::nothrow) relay_handle;
+    if (h == nullptr) return RELAY_ENOMEM;
+    int rc = RELAY_OK;
+    try {
+        rc = relaysum::build_program(n, edges, n_edges, &h->prog);
+    } catch (...) {
+        rc = RELAY_ENOMEM;
+    }
+    if (rc != RELAY_OK) {
+        delete h;
+        return rc;
+    }
+    h->d = d;
+    h->ld = ld;
+    h->nquads = (d + 3) / 4;
+    *out = h;
+    return RELAY_OK;
+}
+
+void relay_destroy(relay_handle* h) { delete h; }
+
+int64_t relay_ld(const relay_handle* h) { return h ? h->ld : RELAY_EINVAL; }
+
+int32_t relay_num_edges(const relay_handle* h) { return h ? h->prog.E : RELAY_EINVAL; }
+
+int relay_edges(const relay_handle* h, int32_t* src, int32_t* dst) {
+    if (!h || (h->prog.E > 0 && (!src || !dst))) return RELAY_EINVAL;
+    for (int e = 0; e < h->prog.E; ++e) {
+        src[e] = h->prog.edge_src[e];
+        dst[e] = h->prog.edge_dst[e];
+    }
+    return RELAY_OK;
+}
+
+int relay_set_rebuild_mode(relay_handle* h, int32_t mode) {
+    if (!h || (mode != 0 && mode != 1)) return RELAY_EINVAL;
+    h->mode = mode;
+    return RELAY_OK;
+}
+
+int relay_set_coord_offset(relay_handle* h, int64_t c0) {
+    if (!h || c0 < 0 || (c0 & 3) != 0) return RELAY_EINVAL;
+    if ((c0 + h->ld) / 4 >= (int64_t(1) << 32)) return RELAY_EINVAL;
+    h->c0 = c0;
+    return RELAY_OK;
+}
+
+int relay_set_objective(relay_handle* h, const float* mu, float sigma) {
+    if (!h || !std::isfinite(sigma) || sigma < 0.0f) return RELAY_EINVAL;
+    if (h->d > 0 && (!mu || !aligned16(mu))) return RELAY_EINVAL;
+    h->mu = mu;
+    h->sigma = sigma;
+    h->has_objective = true;
+    return RELAY_OK;
+}
+
+int relay_fill_objective(relay_handle* h, float* mu, const float* mix, int32_t K, float mu_scale,
+                         uint64_t mu_seed, relay_stream_t stream) {
+    if (!h || K < 0 || !std::isfinite(mu_scale)) return RELAY_EINVAL;
+    if (h->d == 0) return RELAY_OK;
+    if (!mu || !aligned16(mu) || (K > 0 && !mix)) return RELAY_EINVAL;
+    const int threads = 256;
+    relay_fill_mu_kernel<<<grid_for(h->ld / 4, threads), threads, 0, stream>>>(
+        mu, mix, h->prog.n, K, h->ld, h->d, static_cast<uint32_t>(h->c0 / 4), mu_scale,
+        static_cast<uint32_t>(mu_seed), static_cast<uint32_t>(mu_seed >> 32));
+    return launch_status();
+}
+
+int relay_init(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* counts, float x0_std,
+               uint64_t seed, relay_stream_t stream) {
+    if (!h || !std::isfinite(x0_std)) return RELAY_EINVAL;
+    const int E = h->prog.E;
+    if (E > 0 && !counts) return RELAY_EINVAL;
+    if (h->d > 0 && (!x || !aligned16(x) || (E > 0 && (!msg_a || !aligned16(msg_a))) ||
+                     (msg_b && !aligned16(msg_b))))
+        return RELAY_EINVAL;
+    if (E > 0 && cudaMemsetAsync(counts, 0, sizeof(int32_t) * E, stream) != cudaSuccess) return RELAY_ECUDA;
+    if (h->d == 0) return RELAY_OK;
+    const int threads = 256;
+    relay_init_kernel<<<grid_for(h->ld / 4, threads), threads, 0, stream>>>(
+        x, E > 0 ? msg_a : nullptr, E > 0 ? msg_b : nullptr, h->prog.n, E, h->ld, h->d,
+        static_cast<uint32_t>(h->c0 / 4), x0_std, static_cast<uint32_t>(seed),
+        static_cast<uint32_t>(seed >> 32));
+    return launch_status();
+}
+
+int relay_step_counts(relay_handle* h, int32_t* counts, relay_stream_t stream) {
+    if (!h) return RELAY_EINVAL;
+    if (h->prog.E == 0) return RELAY_OK;
+    if (!counts) return RELAY_EINVAL;
+    relay_counts_kernel<<<1, 256, 0, stream>>>(h->prog, counts);
+    return launch_status();
+}
+
+int relay_step_models(relay_handle* h, float* x, const float* msg_in, float* msg_out,
+                      const int32_t* counts, float lr, uint64_t seed, int64_t step,
+                      relay_stream_t stream) {
+    const int rc = check_step_args(h, x, msg_in, msg_out, counts, lr, step);
+    if (rc != RELAY_OK) return rc;
+    if (h->d == 0) return RELAY_OK;
+    ModelArgs a;
+    a.x = x;
+    a.mu = h->mu;
+    a.msg_in = msg_in;
+    a.msg_out = msg_out;
+    a.counts = counts;
+    a.ld = h->ld;
+    a.nquads = h->nquads;
+    a.q0 = static_cast<uint32_t>(h->c0 / 4);
+    a.step = static_cast<uint32_t>(step);
+    a.k0 = static_cast<uint32_t>(seed);
+    a.k1 = static_cast<uint32_t>(seed >> 32);
+    a.lr = lr;
+    a.sigma = h->sigma;
+    return h->mode == 0 ? launch_models<0>(h, a, stream) : launch_models<1>(h, a, stream);
+}
+
+int relay_step(relay_handle* h, float* x, const float* msg_in, float* msg_out, int32_t* counts, float lr,
+               uint64_t seed, int64_t step, relay_stream_t stream) {
+    // every check of relay_step_models runs before the counter launch, so a
+    // rejected step leaves the counters untouched
+    int rc = check_step_args(h, x, msg_in, msg_out, counts, lr, step);
+    if (rc != RELAY_OK) return rc;
+    rc = relay_step_counts(h, counts, stream);
+    if (rc != RELAY_OK) return rc;
+    return relay_step_models(h, x, msg_in, msg_out, counts, lr, seed, step, stream);
+}
+
+int relay_nbar(const relay_handle* h, const int32_t* counts_host, int32_t* nbar_host) {
+    if (!h || !nbar_host || (h->prog.E > 0 && !counts_host)) return RELAY_EINVAL;
+    for (int i = 0; i < h->prog.n; ++i) {
+        const NodeRec& r = h->prog.node[i];
+        int32_t s = 1;
+        for (int p = 0; p < r.deg; ++p) s += counts_host[h->prog.pos_in[r.pos_base + p]];
+        nbar_host[i] = s;
+    }
+    return RELAY_OK;
+}
+
+int relay_program(const relay_handle* h, int32_t* nslots, int32_t* order, int32_t* node_rec,
+                  int32_t* pos_rec) {
+    if (!h) return RELAY_EINVAL;
+    const Program& p = h->prog;
+    if (nslots) *nslots = p.nslots;
+    for (int i = 0; i < p.n; ++i) {
+        if (order) order[i] = p.order[i];
+        if (node_rec) {
+            const NodeRec& r = p.node[i];
+            const int32_t v[8] = {r.deg, r.pos_base, r.parent_pos, r.recv_slot,
+                                  r.acc_slot, r.parent_acc, r.fin_parent, r.parent};
+            std::memcpy(node_rec + 8 * i, v, sizeof(v));
+        }
+    }
+    if (pos_rec)
+        for (int e = 0; e < p.E; ++e) {
+            pos_rec[3 * e] = p.pos_in[e];
+            pos_rec[3 * e + 1] = p.pos_out[e];
+            pos_rec[3 * e + 2] = p.pos_slot[e];
+        }
+    return RELAY_OK;
+}
+
+const char* relay_error_string(int status) {
+    switch (status) {
+        case RELAY_OK: return "ok";
+        case RELAY_EINVAL: return "invalid argument";
+        case RELAY_ENOTTREE: return "edge list is not a tree";
+        case RELAY_ECUDA: return "CUDA launch or runtime error";
+        case RELAY_ENOMEM: return "host allocation failed";
+        case RELAY_EUNSUPPORTED: return "unsupported size";
+        default: return "unknown status";
+    }
+}
+
+}  // extern "C"

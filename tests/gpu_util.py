@@ -1,0 +1,84 @@
+"""Shared helpers of the GPU parity tests: run the CUDA path, run the oracle on
+chosen coordinates, compare with the parity metric.
+
+Parity metric (per array, padding excluded):
+    max_e |g_e - r_e| / max(|r_e|, rms(r))  <=  1e-5
+with g the fp32 GPU value and r the fp64 oracle value; counters must be equal.
+The fp32 path differs from the fp64 definition only by rounding: a float32
+restatement of the step stays within 1e-6 of the oracle on every workload
+(10x below the bar), so 1e-5 leaves room for the GPU's own summation order
+and its fp32 logf/sincospif in the noise.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import paper_2110_04175_gb300 as rs
+from oracle import oracle
+
+RTOL = 1e-5
+
+
+def parity_error(g: np.ndarray, r: np.ndarray) -> float:
+    g = np.asarray(g, dtype=np.float64)
+    r = np.asarray(r, dtype=np.float64)
+    if r.size == 0:
+        return 0.0
+    rms = float(np.sqrt(np.mean(r * r)))
+    denom = np.maximum(np.abs(r), rms if rms > 0 else 1.0)
+    return float(np.max(np.abs(g - r) / denom))
+
+
+def gpu_run(w, steps: int, mode: int | None = None, d: int | None = None, c0: int = 0,
+            stream=None) -> rs.RelayRun:
+    """Runs `steps` RelaySGD steps of workload `w` on cuda:0 through the C ABI."""
+    run = rs.RelayRun(w.n, w.d if d is None else d, w.edges, device="cuda:0",
+                      mode=w.mode if mode is None else mode, c0=c0)
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    for _ in range(steps):
+        run.step(w.lr, w.seed, stream)
+    torch.cuda.synchronize()
+    return run
+
+
+def oracle_range(w, c0: int, length: int, steps: int, mode: int | None = None) -> oracle.State:
+    st = oracle.State(w.n, w.edges, length, c0=c0)
+    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+    st.advance(steps, float(np.float32(w.lr)), float(np.float32(w.sigma)), w.seed,
+               w.mode if mode is None else mode)
+    return st
+
+
+def sample_columns(d: int, head: int, tail: int, n_random: int, seed: int = 0):
+    """Contiguous ranges (start, length) to compare: the first `head`
+    coordinates, the last `tail` (ragged end of the last quad included) and
+    `n_random` single coordinates drawn uniformly."""
+    rng = np.random.default_rng(seed)
+    ranges = [(0, min(head, d))]
+    if d > head:
+        start = max(head, d - tail)
+        ranges.append((start, d - start))
+    for c in rng.choice(np.arange(head, max(head + 1, d - tail)), size=min(n_random, max(0, d - head - tail)),
+                        replace=False):
+        ranges.append((int(c), 1))
+    return ranges
+
+
+def compare_ranges(run: rs.RelayRun, w, ranges, steps: int, mode: int | None = None, c0: int = 0):
+    """Max parity error of x and of the last messages over the given ranges;
+    asserts the counters are bit-exact."""
+    gx, gm, ox, om = [], [], [], []
+    counts = None
+    for start, length in ranges:
+        st = oracle_range(w, c0 + start, length, steps, mode)
+        gx.append(run.x[:, start:start + length].double().cpu().numpy())
+        gm.append(run.messages[:run.E, start:start + length].double().cpu().numpy())
+        ox.append(st.x)
+        om.append(st.msg)
+        counts = st.counts
+    g_counts = run.counts[:run.E].cpu().numpy()
+    assert np.array_equal(g_counts, counts), (g_counts, counts)
+    ex = parity_error(np.concatenate(gx, axis=1), np.concatenate(ox, axis=1))
+    em = parity_error(np.concatenate(gm, axis=1), np.concatenate(om, axis=1)) if run.E else 0.0
+    return ex, em

@@ -1,0 +1,208 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
+
+Counters bit-exact; models and messages within the parity metric of
+tests/gpu_util.py (1e-5).  Small workloads are compared on every coordinate;
+the full-size workloads run in full on the GPU, in the launch configuration
+bench.py times, and are compared on the first and last coordinates (the
+ragged tail included) and on coordinates drawn at random -- every coordinate
+of the method evolves independently and the noise is keyed by the absolute
+coordinate, so the oracle computes those columns exactly as in a full run.
+"""
+import gc
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2110_04175_gb300 as rs
+from oracle import oracle
+from paper_2110_04175_gb300 import build as rs_build
+from paper_2110_04175_gb300 import workloads as wl
+from tests import treeutil as tu
+from tests.gpu_util import RTOL, compare_ranges, gpu_run, oracle_range, parity_error, sample_columns
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    rs_build.build()
+    yield
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+def _free():
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+# ------------------------------------------------------------ random streams
+
+def test_initial_model_and_centres_match_oracle_normals():
+    d = 4096 + 7
+    run = rs.RelayRun(3, d, wl.chain(3), device="cuda:0")
+    mix = np.array([[1, 0, 0], [0, 1, 0], [0.25, 0.5, 0.25]], dtype=np.float32)
+    run.init(1.0, 1234, mix, 1.5, 99, 0.0)
+    torch.cuda.synchronize()
+    x = run.x.double().cpu().numpy()
+    mu = run.mu.double().cpu().numpy()
+    want_x = oracle.fill_x0(3, 1.0, 1234, 0, d)
+    want_mu = oracle.fill_mu(3, mix.astype(np.float64), 1.5, 99, 0, d)
+    assert parity_error(x[:, :d], want_x) < 2e-6
+    assert parity_error(mu[:, :d], want_mu) < 2e-6
+    assert np.all(x[:, d:] == 0) and np.all(mu[:, d:] == 0)
+    assert np.all(run.msg[0].cpu().numpy() == 0) and np.all(run.msg[1].cpu().numpy() == 0)
+
+
+def test_gradient_noise_stream():
+    """n = 1, x = mu = 0, lr = 1: one step gives x^1 = -sigma xi^0 exactly as
+    the oracle's stream-0 normals, at a non-zero coordinate offset too."""
+    for c0, step in ((0, 0), (4096, 7)):
+        run = rs.RelayRun(1, 1000, np.zeros((0, 2), np.int32), device="cuda:0", c0=c0)
+        run.init(0.0, 77, np.zeros((1, 1), np.float32), 0.0, 0, 0.5)
+        run.t = step
+        run.step(1.0, 77)
+        torch.cuda.synchronize()
+        want = -0.5 * oracle.normals(77, c0, 1000, row=0, step=step, stream=0)
+        assert parity_error(run.x[0, :1000].double().cpu().numpy(), want) < 2e-6
+
+
+# ------------------------------------------------------------------ counters
+
+@pytest.mark.parametrize("n", [2, 3, 4, 5, 6])
+def test_counts_bit_exact_all_small_trees(n):
+    trees = list(tu.all_trees(n))
+    rng = np.random.default_rng(n)
+    if len(trees) > 40:
+        trees = [trees[k] for k in rng.choice(len(trees), 40, replace=False)]
+    for edges in trees:
+        h = rs.relay_create(n, 0, edges)
+        E = 2 * (n - 1)
+        counts = torch.zeros(E, dtype=torch.int32, device="cuda:0")
+        want = np.zeros(E, dtype=np.int32)
+        for t in range(tu.diameter(n, edges) + 2):
+            rs.relay_step_counts(h, counts)
+            oracle.run(n, edges, np.zeros((n, 0)), np.zeros((n, 0)), np.zeros((E, 0)), want, 0, 0,
+                       0, t, 1, 0)
+            assert np.array_equal(counts.cpu().numpy(), want)
+
+
+@pytest.mark.parametrize("w", wl.all_workloads(), ids=lambda w: w.name)
+def test_counts_bit_exact_workload_trees(w):
+    h = rs.relay_create(w.n, 0, w.edges)
+    counts = torch.zeros(w.E, dtype=torch.int32, device="cuda:0")
+    want = np.zeros(w.E, dtype=np.int32)
+    steps = tu.diameter(w.n, w.edges.tolist()) + 3
+    for t in range(steps):
+        rs.relay_step_counts(h, counts)
+    oracle.run(w.n, w.edges, np.zeros((w.n, 0)), np.zeros((w.n, 0)), np.zeros((w.E, 0)), want, 0,
+               0, 0, 0, steps, 0)
+    assert np.array_equal(counts.cpu().numpy(), want)
+
+
+# ------------------------------------------------------- full-vector parity
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_chain8_d4096_full_100_steps(mode):
+    """The small workload, every coordinate, 100 steps."""
+    w = wl.chain8_d4096()
+    run = gpu_run(w, w.steps, mode)
+    ex, em = compare_ranges(run, w, [(0, w.d)], w.steps, mode)
+    assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("shape,n,d", [
+    ("single", 1, 4097), ("pair", 2, 33), ("chain", 5, 1), ("chain", 5, 3), ("binary", 7, 5),
+    ("star", 9, 131), ("star", 33, 257), ("random", 23, 1031), ("torus", 16, 4099),
+    ("star", 256, 67), ("chain", 256, 9),
+])
+def test_small_cases_every_coordinate(shape, n, d, mode):
+    """Edge cases: one worker, one edge, d below one quad, ragged tails, the
+    generic high-degree path (stars), the largest supported tree."""
+    edges = {"single": np.zeros((0, 2), np.int32), "pair": wl.chain(2), "chain": wl.chain(n),
+             "binary": wl.binary_tree(n), "star": wl.star(n), "random": wl.random_tree(n, 4),
+             "torus": wl.torus_spanning_tree(4, 4, 2)}[shape]
+    w = wl.Workload(f"{shape}{n}", n, edges, d, wl.identity_mix(n), 1.0, 0.1, 0.1, 0.1, 30)
+    run = gpu_run(w, w.steps, mode)
+    ex, em = compare_ranges(run, w, [(0, d)], w.steps, mode)
+    assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+def test_empty_model_runs_counters_only():
+    run = rs.RelayRun(4, 0, wl.chain(4), device="cuda:0")
+    run.init(0.0, 0, wl.identity_mix(4), 1.0, 0, 0.1)
+    for _ in range(5):
+        run.step(0.1, 0)
+    torch.cuda.synchronize()
+    assert run.counts.cpu().numpy().tolist() == [1, 3, 2, 2, 3, 1]
+
+
+def test_coordinate_offset_slice_equals_full_run():
+    """A handle on coordinates [c0, c0 + len) reproduces those columns of the
+    full vector bit for bit (the multi-GPU sharding over d relies on it)."""
+    w = wl.Workload("bin15", 15, wl.binary_tree(15), 2000, wl.identity_mix(15), 1.0, 0.1, 0.1,
+                    0.1, 20)
+    full = gpu_run(w, w.steps)
+    part = gpu_run(w, w.steps, d=600, c0=800)
+    assert torch.equal(full.x[:, 800:1400], part.x[:, :600])
+    assert torch.equal(full.messages[:, 800:1400], part.messages[:, :600])
+
+
+def test_deterministic_and_resumable():
+    """Two runs are bitwise identical; 10 + 10 steps equal 20 steps."""
+    w = wl.sweep64("torus")
+    w.d = 50_000
+    a = gpu_run(w, 20)
+    b = gpu_run(w, 10)
+    for _ in range(10):
+        b.step(w.lr, w.seed)
+    torch.cuda.synchronize()
+    assert torch.equal(a.x, b.x) and torch.equal(a.messages, b.messages)
+    assert torch.equal(a.counts, b.counts)
+
+
+def test_streams_are_respected():
+    w = wl.chain8_d4096()
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        run = gpu_run(w, 50, stream=s)
+    ref = gpu_run(w, 50)
+    torch.cuda.synchronize()
+    assert torch.equal(run.x, ref.x)
+
+
+# -------------------------------------------------- full-size workloads
+
+FULL = [wl.binary16_resnet20(), wl.chain16_vgg11(), wl.binary32_bert()] + [
+    wl.sweep64(s) for s in ("star", "chain", "binary", "torus")]
+
+
+@pytest.mark.parametrize("w", FULL, ids=lambda w: w.name)
+def test_full_size_workload_sampled(w):
+    """Full d and the workload's step count on the GPU; oracle on the first
+    2048 and last 1031 coordinates and 48 random ones."""
+    _free()
+    run = gpu_run(w, w.steps)
+    ranges = sample_columns(w.d, 2048, 1031, 48, seed=w.n)
+    ex, em = compare_ranges(run, w, ranges, w.steps)
+    del run
+    _free()
+    assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+def test_binary16_resnet20_every_coordinate_mode0():
+    """Alg. 1 rebuild on the ResNet-20-sized vector, all 272,474 coordinates,
+    oracle on every coordinate for the first 10 steps (the warm-up in which
+    nbar < n, where the two rebuild rules differ)."""
+    w = wl.binary16_resnet20()
+    run = gpu_run(w, 10, mode=0)
+    st = oracle_range(w, 0, w.d, 10, 0)
+    gx = run.x[:, :w.d].double().cpu().numpy()
+    gm = run.messages[:w.E, :w.d].double().cpu().numpy()
+    assert parity_error(gx, st.x) <= RTOL
+    assert parity_error(gm, st.msg) <= RTOL
+    assert np.array_equal(run.counts.cpu().numpy(), st.counts)

@@ -1,0 +1,255 @@
+"""CPU checks of the library's host logic (no GPU needed).
+
+The fused kernel follows a visit program built on the host (tree walk,
+shared-memory slot assignment).  Here the program is read back through the
+C ABI and executed in float64 with the kernel's exact sequence of slot reads
+and writes -- every write must land in a free slot, every read in a live
+one -- and the result is compared with the oracle.  A wrong slot assignment,
+parent link or finalisation point fails here before any GPU time is spent.
+"""
+import ctypes
+import re
+
+import numpy as np
+import pytest
+
+import paper_2110_04175_gb300 as rs
+from oracle import oracle
+from paper_2110_04175_gb300 import build as rs_build
+from paper_2110_04175_gb300 import workloads as wl
+from tests import treeutil as tu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    rs_build.build()
+
+
+REG_DEG = 4
+
+
+def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0=0):
+    """One step executed the way relay_counts_kernel + relay_models_kernel do."""
+    nslots, order, node, pos = rs.relay_program(h)
+    E = 2 * (n - 1)
+    src, dst = rs.relay_edges(h)
+    # counters
+    counts = np.zeros(E, dtype=np.int32)
+    for e in range(E):
+        deg, pb = node[src[e]][0], node[src[e]][1]
+        counts[e] = 1 + sum(counts_old[pos[pb + s][0]] for s in range(deg)
+                            if pos[pb + s][0] != (e ^ 1))
+    nbar = [1 + sum(counts[pos[node[i][1] + s][0]] for s in range(node[i][0])) for i in range(n)]
+    if mode == 0:
+        scale = [1.0 / nb for nb in nbar]
+        fill = [0.0] * n
+    else:
+        scale = [1.0 / n] * n
+        fill = [float(n - nb) for nb in nbar]
+    L = x.shape[1]
+    slots = [None] * nslots
+    msg_out = np.full((E, L), np.nan)
+    xnew = np.full((n, L), np.nan)
+    visited = set()
+
+    def write(s, v):
+        assert 0 <= s < nslots and slots[s] is None, f"slot {s} clobbered"
+        slots[s] = v
+
+    def take(s):
+        assert slots[s] is not None, f"slot {s} read while free"
+        v = slots[s]
+        slots[s] = None
+        return v
+
+    def to_parent(rec, out):
+        _, _, _, _, _, pacc, finp, par = rec
+        assert par in visited
+        acc = take(pacc) + out
+        if finp >= 0:
+            assert finp == par
+            xnew[finp] = acc * scale[finp]
+        else:
+            write(pacc, acc)
+
+    for i in order:
+        visited.add(i)
+        rec = node[i]
+        deg, pb, ppos, recv, accs = rec[0], rec[1], rec[2], rec[3], rec[4]
+        z = oracle.normals(seed, c0, L, i, step, 0)
+        xh = x[i] - lr * ((x[i] - mu[i]) + sigma * z)
+        acc = xh.copy()
+        if mode == 1:
+            acc = fill[i] * x[i] + xh
+        if recv >= 0:
+            acc = acc + take(recv)
+        if 0 < deg <= REG_DEG:
+            m = [msg_in[pos[pb + s][0]] for s in range(deg)]
+            for s in range(deg):
+                out = xh + sum((m[r] for r in range(deg) if r != s), np.zeros(L))
+                msg_out[pos[pb + s][1]] = out
+                if s == ppos:
+                    to_parent(rec, out)
+                else:
+                    write(pos[pb + s][2], out)
+        elif deg > REG_DEG:
+            suf = np.zeros(L)
+            for s in range(deg - 1, -1, -1):
+                suf = msg_in[pos[pb + s][0]] + suf
+                write(pos[pb + s][2], suf)
+            pre = xh.copy()
+            for s in range(deg):
+                out = pre if s == deg - 1 else pre + slots[pos[pb + s + 1][2]]
+                pre = pre + msg_in[pos[pb + s][0]]
+                msg_out[pos[pb + s][1]] = out
+                if s == ppos:
+                    take(pos[pb + s][2])
+                    to_parent(rec, out)
+                else:
+                    take(pos[pb + s][2])
+                    write(pos[pb + s][2], out)
+        if accs < 0:
+            xnew[i] = acc * scale[i]
+        else:
+            write(accs, acc)
+    assert all(s is None for s in slots), "slots left live after the walk"
+    assert not np.isnan(xnew).any() and not np.isnan(msg_out).any()
+    return xnew, msg_out, counts, nslots
+
+
+def check_tree(n, edges, mode, steps=3, L=3, seed=1):
+    h = rs.relay_create(n, L, edges)
+    rng = np.random.default_rng(n)
+    mu = rng.normal(size=(n, L))
+    x = np.tile(rng.normal(size=L), (n, 1))
+    E = 2 * (n - 1)
+    st = oracle.State(n, edges, L)
+    st.x = x.copy()
+    st.mu = mu.copy()
+    msg = np.zeros((E, L))
+    counts = np.zeros(E, dtype=np.int32)
+    for t in range(steps):
+        x, msg, counts, nslots = run_program(h, n, x, mu, msg, counts, 0.3, 0.2, seed, t, mode)
+        st.advance(1, 0.3, 0.2, seed, mode)
+        assert np.array_equal(counts, st.counts)
+        assert np.allclose(x, st.x, rtol=1e-12, atol=1e-12)
+        assert np.allclose(msg, st.msg, rtol=1e-12, atol=1e-12)
+    return nslots
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("n", [1, 2, 3, 4, 5, 6])
+def test_program_matches_oracle_small_trees(n, mode):
+    trees = list(tu.all_trees(n))
+    rng = np.random.default_rng(n)
+    if len(trees) > 80:
+        trees = [trees[k] for k in rng.choice(len(trees), 80, replace=False)]
+    for edges in trees:
+        check_tree(n, edges, mode)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("shape", ["star", "chain", "binary", "torus", "random40", "star9"])
+def test_program_matches_oracle_workload_trees(shape, mode):
+    trees = {"star": wl.star(64), "chain": wl.chain(64), "binary": wl.binary_tree(64),
+             "torus": wl.torus_spanning_tree(8, 8, 0), "random40": wl.random_tree(40, 9),
+             "star9": wl.star(9, hub=4)}
+    edges = trees[shape]
+    n = int(edges.max()) + 1
+    check_tree(n, edges, mode, steps=2, L=2)
+
+
+def test_slot_counts_of_workload_trees():
+    """The walk keeps the shared-memory footprint small: O(1) on chains,
+    O(depth) on balanced trees, the hub degree on a star."""
+    def slots(edges):
+        n = int(edges.max()) + 1
+        return rs.relay_program(rs.relay_create(n, 4, edges))[0]
+    assert slots(wl.chain(64)) <= 3
+    assert slots(wl.binary_tree(64)) <= 14
+    assert slots(wl.binary_tree(32)) <= 12
+    assert slots(wl.star(64)) <= 65
+    assert slots(wl.torus_spanning_tree(8, 8, 0)) <= 20
+
+
+# ------------------------------------------------------------ ABI surface
+
+def _declared_functions():
+    import os
+    hdr = os.path.join(rs_build.INCLUDE, "relaysum.h")
+    text = open(hdr).read()
+    return sorted(set(re.findall(r"\b(relay_[a-z_]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol():
+    lib = ctypes.CDLL(rs.library_path())
+    names = _declared_functions()
+    assert "relay_step" in names and "relay_create" in names and len(names) >= 15
+    for name in names:
+        assert hasattr(lib, name), name
+
+
+@pytest.mark.parametrize("edges,n,status", [
+    ([(0, 1), (1, 2), (2, 0)], 3, rs.RELAY_ENOTTREE),
+    ([(0, 1), (0, 1)], 3, rs.RELAY_ENOTTREE),
+    ([(0, 0)], 2, rs.RELAY_ENOTTREE),
+    ([(0, 1), (1, 5)], 3, rs.RELAY_ENOTTREE),
+    ([(0, 1)], 3, rs.RELAY_ENOTTREE),
+    ([], 0, rs.RELAY_EINVAL),
+])
+def test_create_rejects_bad_trees(edges, n, status):
+    with pytest.raises(rs.RelayError) as e:
+        rs.relay_create(n, 8, edges)
+    assert e.value.status == status
+
+
+def test_create_limits_and_layout():
+    with pytest.raises(rs.RelayError) as e:
+        rs.relay_create(rs.RELAY_MAX_N + 1, 8, wl.chain(rs.RELAY_MAX_N + 1))
+    assert e.value.status == rs.RELAY_EUNSUPPORTED
+    with pytest.raises(rs.RelayError):
+        rs.relay_create(2, -1, [(0, 1)])
+    h = rs.relay_create(rs.RELAY_MAX_N, 5, wl.star(rs.RELAY_MAX_N))
+    assert rs.relay_num_edges(h) == 2 * (rs.RELAY_MAX_N - 1)
+    for d, ld in ((0, 0), (1, 32), (32, 32), (33, 64), (272_474, 272_480)):
+        assert rs.relay_ld(rs.relay_create(2, d, [(0, 1)])) == ld
+    src, dst = rs.relay_edges(rs.relay_create(4, 8, [(2, 0), (0, 1), (1, 3)]))
+    assert list(zip(src, dst)) == tu.directed([(2, 0), (0, 1), (1, 3)])
+    h = rs.relay_create(3, 8, [(0, 1), (1, 2)])
+    with pytest.raises(rs.RelayError):
+        rs.relay_set_rebuild_mode(h, 2)
+    with pytest.raises(rs.RelayError):
+        rs.relay_set_coord_offset(h, 6)
+    rs.relay_set_coord_offset(h, 8)
+
+
+def test_nbar_host_helper_matches_closed_form():
+    edges = wl.binary_tree(7)
+    h = rs.relay_create(7, 4, edges)
+    counts = np.zeros(12, dtype=np.int32)
+    oracle.run(7, edges, np.zeros((7, 0)), np.zeros((7, 0)), np.zeros((12, 0)), counts, 0, 0, 0,
+               0, 10, 0)
+    assert np.array_equal(rs.relay_nbar(h, counts), np.full(7, 7))
+
+
+def test_step_rejects_bad_arguments_before_any_launch():
+    """Argument checks run on the host before anything touches a device, so
+    they are testable without a GPU (the pointers below are never used)."""
+    h = rs.relay_create(3, 64, wl.chain(3))
+    lib = ctypes.CDLL(rs.library_path())
+    lib.relay_step.argtypes = [ctypes.c_void_p] * 5 + [ctypes.c_float, ctypes.c_uint64,
+                                                       ctypes.c_int64, ctypes.c_void_p]
+    fake = 0x10000
+    # no objective bound yet
+    assert lib.relay_step(h.raw, fake, fake * 2, fake * 3, fake * 4, 0.1, 0, 0, None) == rs.RELAY_EINVAL
+    lib.relay_set_objective.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_float]
+    assert lib.relay_set_objective(h.raw, fake, 0.1) == rs.RELAY_OK
+    assert lib.relay_set_objective(h.raw, fake + 4, 0.1) == rs.RELAY_EINVAL  # misaligned
+    assert lib.relay_set_objective(h.raw, fake, -1.0) == rs.RELAY_EINVAL
+    big = 1 << 30
+    # msg_in == msg_out, negative step, non-finite lr, overlapping x/messages
+    assert lib.relay_step(h.raw, fake, big, big, fake, 0.1, 0, 0, None) == rs.RELAY_EINVAL
+    assert lib.relay_step(h.raw, fake, big, 2 * big, fake, 0.1, 0, -1, None) == rs.RELAY_EINVAL
+    assert lib.relay_step(h.raw, fake, big, 2 * big, fake, float("nan"), 0, 0, None) == rs.RELAY_EINVAL
+    assert lib.relay_step(h.raw, fake, fake + 256, 2 * big, fake, 0.1, 0, 0, None) == rs.RELAY_EINVAL
+    assert lib.relay_step(h.raw, fake, big, 2 * big, fake, 0.1, 0, 1 << 32, None) == rs.RELAY_EINVAL
