@@ -1,0 +1,74 @@
+"""World-size-2 checks of the multi-GPU host logic on CPU (gloo).
+
+bench.py shards the model vector over ranks by coordinate: rank r owns the
+slice starting at shard_offset(r, d) of one longer vector, with no data-path
+collective; the job time is the max over ranks.  Here two gloo ranks run the
+oracle on their slices and check that the gathered result equals one
+unsharded run, and that the max-reduction and barrier behave.
+"""
+import os
+import socket
+
+import numpy as np
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, result_dir):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        import bench
+        from oracle import oracle
+        from paper_2110_04175_gb300 import workloads as wl
+
+        # max over ranks
+        got = bench.reduce_max(float(rank + 1) * 1.5, world)
+        assert got == 1.5 * world
+        bench.barrier(world)
+
+        # d-sharding: each rank runs its slice of a longer vector
+        w = wl.Workload("bin7", 7, wl.binary_tree(7), 10, wl.identity_mix(7), 1.0, 0.1, 0.1,
+                        0.1, 6)
+        c0 = bench.shard_offset(rank, w.d)
+        st = oracle.State(w.n, w.edges, w.d, c0=c0)
+        st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+        st.advance(w.steps, w.lr, w.sigma, w.seed, w.mode)
+        mine = torch.from_numpy(st.x.copy())
+        parts = [torch.zeros_like(mine) for _ in range(world)]
+        dist.all_gather(parts, mine)
+        if rank == 0:
+            stride = bench.shard_offset(1, w.d)
+            full = oracle.State(w.n, w.edges, stride * world)
+            full.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+            full.advance(w.steps, w.lr, w.sigma, w.seed, w.mode)
+            for r in range(world):
+                want = full.x[:, r * stride: r * stride + w.d]
+                assert np.array_equal(parts[r].numpy(), want)
+            open(os.path.join(result_dir, "ok"), "w").write("ok")
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_ranks_shard_over_d_and_reduce_max(tmp_path):
+    port = _free_port()
+    mp.spawn(_worker, args=(2, port, str(tmp_path)), nprocs=2, join=True)
+    assert (tmp_path / "ok").exists()
+
+
+def test_shard_offsets_are_quad_aligned():
+    import bench
+    for d in (1, 3, 4, 5, 110_000_000, 9_231_114):
+        for r in range(8):
+            c0 = bench.shard_offset(r, d)
+            assert c0 % 4 == 0 and c0 >= r * d
+            assert bench.shard_offset(r + 1, d) - c0 >= d
