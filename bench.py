@@ -316,6 +316,36 @@ def run_native(args, w, rank: int, world: int):
     print(json.dumps(line), flush=True)
 
 
+def host_mem_available() -> int:
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
+
+
+def pinned_like(t):
+    """A page-locked host tensor shaped like `t` (registered in place with
+    cudaHostRegister, so no power-of-two rounding of the pinned pool)."""
+    import torch
+    h = torch.empty(t.shape, dtype=t.dtype)
+    cudart = torch.cuda.cudart()
+    rc = cudart.cudaHostRegister(h.data_ptr(), h.numel() * h.element_size(), 0)
+    if int(rc) != 0:
+        raise RuntimeError(f"cudaHostRegister failed ({rc})")
+    return h
+
+
+def unpin(*tensors):
+    import torch
+    cudart = torch.cuda.cudart()
+    for t in tensors:
+        cudart.cudaHostUnregister(t.data_ptr())
+
+
 def run_e2e(args, w, run, dev, stream, world: int):
     """relay_step with x, messages and counters living in pinned host memory:
     every step copies them to the device, runs, and copies the results back."""
@@ -323,36 +353,48 @@ def run_e2e(args, w, run, dev, stream, world: int):
 
     import paper_2110_04175_gb300 as rs
 
-    hx = torch.empty_like(run.x, device="cpu").pin_memory()
-    hm_in = torch.empty_like(run.msg[0], device="cpu").pin_memory()
-    hm_out = torch.empty_like(run.msg[0], device="cpu").pin_memory()
-    hc = torch.empty_like(run.counts, device="cpu").pin_memory()
-    hx.copy_(run.x)
-    hm_in.copy_(run.msg[run.cur])
-    hc.copy_(run.counts)
-    torch.cuda.synchronize(dev)
-    h2d = (hx.numel() + hm_in.numel() + hc.numel()) * 4
-    d2h = (hx.numel() + hm_out.numel() + hc.numel()) * 4
-    barrier(world)
-    start = torch.cuda.Event(enable_timing=True)
-    end = torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    for _ in range(args.e2e_steps):
-        run.x.copy_(hx, non_blocking=True)
-        run.msg[0].copy_(hm_in, non_blocking=True)
-        run.counts.copy_(hc, non_blocking=True)
-        rs.relay_step(run.h, run.x, run.msg[0], run.msg[1], run.counts, w.lr, w.seed, run.t, stream)
-        hx.copy_(run.x, non_blocking=True)
-        hm_out.copy_(run.msg[1], non_blocking=True)
-        hc.copy_(run.counts, non_blocking=True)
-        run.t += 1
-        hm_in, hm_out = hm_out, hm_in
-    end.record(stream)
-    torch.cuda.synchronize(dev)
-    ms = reduce_max(start.elapsed_time(end), world)
+    need = (run.x.numel() + 2 * run.msg[0].numel() + run.counts.numel()) * 4
+    avail = host_mem_available()
+    if need > 0.6 * avail:
+        return {"value": None, "unit": "steps/s",
+                "skipped": f"pinned host state of {need / 1e9:.1f} GB exceeds 60% of the "
+                           f"{avail / 1e9:.1f} GB available"}
+    hx = pinned_like(run.x)
+    hm_in = pinned_like(run.msg[0])
+    hm_out = pinned_like(run.msg[0])
+    hc = pinned_like(run.counts)
+    try:
+        hx.copy_(run.x)
+        hm_in.copy_(run.msg[run.cur])
+        hc.copy_(run.counts)
+        torch.cuda.synchronize(dev)
+        h2d = (hx.numel() + hm_in.numel() + hc.numel()) * 4
+        d2h = (hx.numel() + hm_out.numel() + hc.numel()) * 4
+        barrier(world)
+        start = torch.cuda.Event(enable_timing=True)
+        end = torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for _ in range(args.e2e_steps):
+            run.x.copy_(hx, non_blocking=True)
+            run.msg[0].copy_(hm_in, non_blocking=True)
+            run.counts.copy_(hc, non_blocking=True)
+            rs.relay_step(run.h, run.x, run.msg[0], run.msg[1], run.counts, w.lr, w.seed, run.t,
+                          stream)
+            hx.copy_(run.x, non_blocking=True)
+            hm_out.copy_(run.msg[1], non_blocking=True)
+            hc.copy_(run.counts, non_blocking=True)
+            run.t += 1
+            hm_in, hm_out = hm_out, hm_in
+        end.record(stream)
+        torch.cuda.synchronize(dev)
+        ms = reduce_max(start.elapsed_time(end), world)
+    finally:
+        torch.cuda.synchronize(dev)
+        unpin(hx, hm_in, hm_out, hc)
     return {"value": round(world * args.e2e_steps / (ms / 1e3), 4), "unit": "steps/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
-            "path": "relay_step with x, messages and counters in pinned host memory"}
+            "path": "relay_step with x, messages and counters in pinned host memory, "
+                    "copied in and out every step"}
 
 
 def traffic_per_launch(w):
@@ -375,12 +417,17 @@ def main(argv=None):
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     p.add_argument("--e2e-steps", type=int, default=3)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--d", type=int, default=None,
+                   help="override the workload's d (small cases for profiling; not a bench line)")
     args = p.parse_args(argv)
     if args.warmup < 3:
         p.error("--warmup must be >= 3")
 
     from paper_2110_04175_gb300 import workloads as wl
     w = wl.by_name(args.workload)
+    if args.d is not None:
+        w.d = args.d
+        w.name = f"{w.name}@d={args.d}"
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if args.impl == "reference":
