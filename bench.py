@@ -167,15 +167,16 @@ def oracle_sample(w, seconds: float = 15.0, max_len: int = 1 << 20):
     workload `w`, scaled to steps/s of the full d."""
     import numpy as np
     from oracle import oracle
+    edges = w.edges[0] if isinstance(w.edges, list) else w.edges  # a sample in the first window
     length = 2048
-    st = oracle.State(w.n, w.edges, length)
+    st = oracle.State(w.n, edges, length)
     st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
     t0 = time.perf_counter()
     st.advance(1, w.lr, w.sigma, w.seed, w.mode)
     per_coord_step = (time.perf_counter() - t0) / length
     steps = 4
     length = int(min(max_len, w.d, max(1024, seconds / (steps * per_coord_step))))
-    st = oracle.State(w.n, w.edges, length)
+    st = oracle.State(w.n, edges, length)
     st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
     t0 = time.perf_counter()
     st.advance(steps, w.lr, w.sigma, w.seed, w.mode)
@@ -192,15 +193,16 @@ def run_reference(args, w, rank: int):
     from oracle import oracle
     if rank != 0:
         return
+    edges = w.edges[0] if isinstance(w.edges, list) else w.edges  # a sample in the first window
     length = 4096
-    st = oracle.State(w.n, w.edges, length)
+    st = oracle.State(w.n, edges, length)
     st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
     t0 = time.perf_counter()
     st.advance(1, w.lr, w.sigma, w.seed, w.mode)
     per_coord = (time.perf_counter() - t0) / length
     budget = 90.0 / max(1, args.steps + args.warmup)
     length = int(max(256, min(1 << 20, w.d, budget / per_coord)))
-    st = oracle.State(w.n, w.edges, length)
+    st = oracle.State(w.n, edges, length)
     st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
     st.advance(args.warmup, w.lr, w.sigma, w.seed, w.mode)
     t0 = time.perf_counter()
@@ -223,7 +225,8 @@ def run_reference(args, w, rank: int):
 
 def workload_config(w, gpus: int) -> dict:
     shape = {"binary": "balanced binary tree (heap order)", "chain": "chain", "star": "star",
-             "torus": "uniform spanning tree of the 8x8 torus"}
+             "torus": "uniform spanning tree of the 8x8 torus",
+             "double": "double binary trees (two complementary trees, half the coordinates each)"}
     kind = next((v for k, v in shape.items() if w.name.startswith(k)), w.name)
     return {"workload": w.name, "n_workers": w.n, "tree": kind, "d": w.d, "directed_edges": w.E,
             "rebuild": "robust (Section 4.4)" if w.mode == 1 else "Algorithm 1",
@@ -246,26 +249,29 @@ def run_native(args, w, rank: int, world: int):
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
     c0 = shard_offset(rank, w.d)
-    run = rs.RelayRun(w.n, w.d, w.edges, device=dev, mode=w.mode, c0=c0)
+    run = rs.RelayRun(w.n, w.d, w.edges, device=dev, mode=w.mode, c0=c0, objective=args.objective)
     run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
     h = run.h
 
     def one_step(ev=None):
-        if ev is not None:
-            ev[0].record(stream)
-        rs.relay_step_counts(h, run.counts, stream)
-        if ev is not None:
-            ev[1].record(stream)
-        rs.relay_step_models(h, run.x, run.msg[run.cur], run.msg[1 - run.cur], run.counts, w.lr,
-                             w.seed, run.t, stream)
-        if ev is not None:
-            ev[2].record(stream)
-        run.cur = 1 - run.cur
+        for k, tr in enumerate(run.trees):
+            if ev is not None:
+                ev[k][0].record(stream)
+            rs.relay_step_counts(tr.h, tr.counts, stream)
+            if ev is not None:
+                ev[k][1].record(stream)
+            rs.relay_step_models(tr.h, run._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts,
+                                 w.lr, w.seed, run.t, stream)
+            if ev is not None:
+                ev[k][2].record(stream)
+            tr.cur = 1 - tr.cur
         run.t += 1
 
+    T = len(run.trees)
     for _ in range(args.warmup):
         one_step()
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(T)]
+              for _ in range(args.steps)]
     torch.cuda.synchronize(dev)
     barrier(world)
     torch.cuda.synchronize(dev)
@@ -275,8 +281,10 @@ def run_native(args, w, rank: int, world: int):
         torch.cuda.synchronize(dev)
     barrier(world)
     torch.cuda.synchronize(dev)
-    total_ms = events[0][0].elapsed_time(events[-1][2])
-    models_ms = [events[k][1].elapsed_time(events[k][2]) for k in range(args.steps)]
+    total_ms = events[0][0][0].elapsed_time(events[-1][-1][2])
+    # fused-kernel time per step (one launch per tree)
+    models_ms = [sum(events[k][j][1].elapsed_time(events[k][j][2]) for j in range(T))
+                 for k in range(args.steps)]
     total_ms = reduce_max(total_ms, world)
     steps_per_s = world * args.steps / (total_ms / 1e3)
 
@@ -293,14 +301,15 @@ def run_native(args, w, rank: int, world: int):
     peak = peak or FALLBACK_HBM_GBS
     mean_models_ms = statistics.mean(models_ms)
     alg_bytes = w.bytes_per_step()
+    moved = alg_bytes if args.objective == "generated" else w.bytes_per_step_with_mu()
     achieved = alg_bytes / (mean_models_ms / 1e3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                "frac": round(achieved / peak, 4), "traffic": traffic_per_launch(w),
+                "frac": round(achieved / peak, 4), "traffic": traffic_per_launch(w, args.objective),
                 "kernel": "relay_models_kernel", "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": alg_bytes,
-                "bytes_per_launch_incl_mu": w.bytes_per_step_with_mu(),
-                "achieved_incl_mu": round(w.bytes_per_step_with_mu() / (mean_models_ms / 1e3) / 1e9,
-                                          1),
+                "objective": args.objective,
+                "design_bytes_per_launch": moved,
+                "achieved_design_bytes": round(moved / (mean_models_ms / 1e3) / 1e9, 1),
                 "launch_ms_mean": round(mean_models_ms, 4),
                 "launch_ms_min": round(min(models_ms), 4)}
     cpu = None
@@ -311,7 +320,7 @@ def run_native(args, w, rank: int, world: int):
             "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": workload_config(w, world), "roofline": roofline, "cpu_baseline": cpu,
-            "e2e": e2e, "gpu_launches": 2 * args.steps, "clocks": clocks.summary(),
+            "e2e": e2e, "gpu_launches": 2 * T * args.steps, "clocks": clocks.summary(),
             "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1)}
     print(json.dumps(line), flush=True)
 
@@ -328,22 +337,9 @@ def host_mem_available() -> int:
 
 
 def pinned_like(t):
-    """A page-locked host tensor shaped like `t` (registered in place with
-    cudaHostRegister, so no power-of-two rounding of the pinned pool)."""
+    """A page-locked host tensor shaped like `t` (torch's pinned allocator)."""
     import torch
-    h = torch.empty(t.shape, dtype=t.dtype)
-    cudart = torch.cuda.cudart()
-    rc = cudart.cudaHostRegister(h.data_ptr(), h.numel() * h.element_size(), 0)
-    if int(rc) != 0:
-        raise RuntimeError(f"cudaHostRegister failed ({rc})")
-    return h
-
-
-def unpin(*tensors):
-    import torch
-    cudart = torch.cuda.cudart()
-    for t in tensors:
-        cudart.cudaHostUnregister(t.data_ptr())
+    return torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
 
 
 def run_e2e(args, w, run, dev, stream, world: int):
@@ -353,7 +349,13 @@ def run_e2e(args, w, run, dev, stream, world: int):
 
     import paper_2110_04175_gb300 as rs
 
-    need = (run.x.numel() + 2 * run.msg[0].numel() + run.counts.numel()) * 4
+    if len(run.trees) > 1:
+        return {"value": None, "unit": "steps/s",
+                "skipped": "host-buffer path measured on single-tree workloads"}
+
+    def pow2(b):  # the pinned allocator rounds every block up to a power of two
+        return 1 << max(0, int(b - 1).bit_length())
+    need = pow2(run.x.numel() * 4) + 2 * pow2(run.msg[0].numel() * 4) + pow2(run.counts.numel() * 4)
     avail = host_mem_available()
     if need > 0.6 * avail:
         return {"value": None, "unit": "steps/s",
@@ -390,20 +392,20 @@ def run_e2e(args, w, run, dev, stream, world: int):
         ms = reduce_max(start.elapsed_time(end), world)
     finally:
         torch.cuda.synchronize(dev)
-        unpin(hx, hm_in, hm_out, hc)
+        del hx, hm_in, hm_out, hc
     return {"value": round(world * args.e2e_steps / (ms / 1e3), 4), "unit": "steps/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
             "path": "relay_step with x, messages and counters in pinned host memory, "
                     "copied in and out every step"}
 
 
-def traffic_per_launch(w):
+def traffic_per_launch(w, objective: str):
     """DRAM bytes per launch of the fused kernel from the committed ncu
-    summary for this workload, if one exists (None otherwise)."""
+    summary for this workload and objective source, if one exists."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
-            return json.load(f).get(w.name)
+            return json.load(f).get(f"{w.name}/{objective}")
     except (OSError, ValueError):
         return None
 
@@ -417,6 +419,8 @@ def main(argv=None):
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     p.add_argument("--e2e-steps", type=int, default=3)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--objective", choices=["generated", "stored"], default="stored",
+                   help="regenerate the centres mu in the kernel, or read a stored mu array")
     p.add_argument("--d", type=int, default=None,
                    help="override the workload's d (small cases for profiling; not a bench line)")
     args = p.parse_args(argv)

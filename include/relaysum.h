@@ -20,8 +20,10 @@
  * Conventions shared by every call:
  *   - Layout.  x and mu are fp32 [n][ld], messages fp32 [E][ld] with
  *     E = 2(n-1), counters int32 [E]; ld = relay_ld(h) >= d is the padded
- *     row stride (a multiple of 32 floats).  Columns [d, ld) are padding:
- *     the library zeroes them on init and never reads them as data.
+ *     row stride (a multiple of 32 floats; relay_set_strides sets others).
+ *     The kernels touch columns [0, 4 ceil(d/4)) of each row only; init
+ *     zeroes the ragged columns [d, 4 ceil(d/4)), whose values after a step
+ *     are unspecified, and never reads or writes columns beyond.
  *     Undirected edge u of the edge list gives directed edges 2u
  *     (edges[2u] -> edges[2u+1]) and 2u+1 (the reverse).
  *   - Ownership.  The caller allocates and owns every device buffer; a
@@ -84,6 +86,13 @@ int32_t relay_num_edges(const relay_handle *h);
  * Edge 2u is edges[u][0] -> edges[u][1], edge 2u+1 its reverse. */
 int relay_edges(const relay_handle *h, int32_t *src, int32_t *dst);
 
+/* Row strides (floats) of x / mu and of the message buffers, for a handle
+ * working on a column window of wider arrays (for example the two trees of
+ * a double binary tree, each owning half the coordinates of one model
+ * array).  Each must be a multiple of 4 and >= 4 ceil(d / 4); pointers
+ * passed to later calls must stay 16-byte aligned.  Default: relay_ld(h). */
+int relay_set_strides(relay_handle *h, int64_t ld_x, int64_t ld_msg);
+
 /* Rebuild rule: 0 = Algorithm 1 (divide by nbar), 1 = robust rule of
  * Section 4.4 (fill the n - nbar missing models with x_i^t, divide by n).
  * The default is 1. */
@@ -100,17 +109,27 @@ int relay_set_coord_offset(relay_handle *h, int64_t c0);
  * valid while steps using it run), sigma >= 0 the gradient-noise std. */
 int relay_set_objective(relay_handle *h, const float *mu, float sigma);
 
+/* Binds the same objective without a mu array: the fused kernel regenerates
+ * mu_i(c) = mu_scale * sum_k mix[i][k] N_k(c) on the fly (Gaussian centres
+ * N_k from Philox stream 1, row k), bit-identical to what
+ * relay_fill_objective writes, so a step reads 4 n d fewer bytes.  mix is a
+ * HOST fp32 [n][K] matrix, copied (its non-zeros) into the handle; sigma >= 0
+ * the gradient-noise std.  RELAY_EUNSUPPORTED if mix has more than 1024
+ * non-zeros. */
+int relay_set_objective_generated(relay_handle *h, const float *mix, int32_t K, float mu_scale,
+                                  uint64_t mu_seed, float sigma);
+
 /* Fills mu (device fp32 [n][ld]) with mu_i(c) = mu_scale * sum_k
  * mix[i][k] N_k(c): K Gaussian centres N_k (Philox stream 1, row k) mixed by
  * the device fp32 [n][K] matrix `mix` (identity for one centre per worker,
- * Dirichlet rows for a mixture).  Padding columns are set to 0. */
+ * Dirichlet rows for a mixture). */
 int relay_fill_objective(relay_handle *h, float *mu, const float *mix, int32_t K,
                          float mu_scale, uint64_t mu_seed, relay_stream_t stream);
 
 /* Initial state of Algorithm 1: x_i^0 = x0_std * N(c) for every worker (one
  * shared draw, Philox stream 2), m^{-1} = 0 in msg_a (and in msg_b unless it
  * is NULL), c^{-1} = 0.  x: device [n][ld]; msg_a, msg_b: device [E][ld];
- * counts: device int32 [E].  Padding columns are set to 0. */
+ * counts: device int32 [E]. */
 int relay_init(relay_handle *h, float *x, float *msg_a, float *msg_b, int32_t *counts,
                float x0_std, uint64_t seed, relay_stream_t stream);
 
@@ -142,10 +161,10 @@ int relay_nbar(const relay_handle *h, const int32_t *counts_host, int32_t *nbar_
 
 /* Introspection of the fused kernel's visit program (for tests and tools):
  * number of shared-memory accumulator slots per thread, the visit order
- * (int32 [n]), per node 8 ints {deg, pos_base, parent_pos, recv_slot,
- * acc_slot, parent_acc, fin_parent, parent} (int32 [n][8]) and per
- * position 3 ints {in_edge, out_edge, slot} (int32 [E][3]); any output
- * pointer may be NULL. */
+ * (int32 [n]), per node 10 ints {deg, pos_base, parent_pos, recv_slot,
+ * acc_slot, parent_acc, fin_parent, parent, tot_slot, flags} (int32 [n][10];
+ * flags bit 0: recv_slot holds the parent's total) and per position 3 ints
+ * {in_edge, out_edge, slot} (int32 [E][3]); any output pointer may be NULL. */
 int relay_program(const relay_handle *h, int32_t *nslots, int32_t *order, int32_t *node_rec,
                   int32_t *pos_rec);
 

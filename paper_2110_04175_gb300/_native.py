@@ -44,8 +44,10 @@ def _load():
             "relay_num_edges": (i32, [vp]),
             "relay_edges": (ctypes.c_int, [vp, vp, vp]),
             "relay_set_rebuild_mode": (ctypes.c_int, [vp, i32]),
+            "relay_set_strides": (ctypes.c_int, [vp, i64, i64]),
             "relay_set_coord_offset": (ctypes.c_int, [vp, i64]),
             "relay_set_objective": (ctypes.c_int, [vp, vp, f32]),
+            "relay_set_objective_generated": (ctypes.c_int, [vp, vp, i32, f32, u64, f32]),
             "relay_fill_objective": (ctypes.c_int, [vp, vp, vp, i32, f32, u64, vp]),
             "relay_init": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, vp]),
             "relay_step_counts": (ctypes.c_int, [vp, vp, vp]),
@@ -163,12 +165,24 @@ def relay_set_rebuild_mode(h, mode: int):
     _check(_load().relay_set_rebuild_mode(_h(h), int(mode)), "relay_set_rebuild_mode")
 
 
+def relay_set_strides(h, ld_x: int, ld_msg: int):
+    _check(_load().relay_set_strides(_h(h), int(ld_x), int(ld_msg)), "relay_set_strides")
+
+
 def relay_set_coord_offset(h, c0: int):
     _check(_load().relay_set_coord_offset(_h(h), int(c0)), "relay_set_coord_offset")
 
 
 def relay_set_objective(h, mu, sigma: float):
     _check(_load().relay_set_objective(_h(h), _ptr(mu), float(sigma)), "relay_set_objective")
+
+
+def relay_set_objective_generated(h, mix, K: int, mu_scale: float, mu_seed: int, sigma: float):
+    """mix: host float32 [n][K] (numpy); the kernel regenerates mu from it."""
+    m = np.ascontiguousarray(np.asarray(mix, dtype=np.float32))
+    _check(_load().relay_set_objective_generated(_h(h), m.ctypes.data if m.size else None, int(K),
+                                                 float(mu_scale), int(mu_seed), float(sigma)),
+           "relay_set_objective_generated")
 
 
 def relay_fill_objective(h, mu, mix, K: int, mu_scale: float, mu_seed: int, stream=None):
@@ -208,57 +222,131 @@ def relay_nbar(h, counts_host) -> np.ndarray:
 
 
 def relay_program(h):
-    """(nslots, order[n], node_rec[n][8], pos_rec[E][3]) of the fused kernel's visit program."""
+    """(nslots, order[n], node_rec[n][10], pos_rec[E][3]) of the fused kernel's visit program."""
     n, E = h.n, relay_num_edges(h)
     nslots = ctypes.c_int32()
     order = np.zeros(n, dtype=np.int32)
-    node = np.zeros((n, 8), dtype=np.int32)
+    node = np.zeros((n, 10), dtype=np.int32)
     pos = np.zeros((max(E, 1), 3), dtype=np.int32)
     _check(_load().relay_program(_h(h), ctypes.addressof(nslots), order.ctypes.data,
                                  node.ctypes.data, pos.ctypes.data), "relay_program")
     return int(nslots.value), order, node, pos[:E]
 
 
-class RelayRun:
-    """Device state of one RelaySGD run, allocated with torch on `device`.
+class _TreeState:
+    """One tree of a run: its handle, column window, messages and counters."""
 
-    Buffers: x [n][ld], mu [n][ld], two message buffers [E][ld] (double
-    buffering), counts int32 [E].  ``step()`` enqueues one relay_step on the
-    current torch stream and swaps the message buffers.
-    """
-
-    def __init__(self, n: int, d: int, edges, device="cuda", mode: int = 1, c0: int = 0):
-        import torch
-        self.h = relay_create(n, d, edges)
-        relay_set_rebuild_mode(self.h, mode)
-        relay_set_coord_offset(self.h, c0)
-        self.n, self.d, self.E, self.ld = n, d, relay_num_edges(self.h), relay_ld(self.h)
-        self.device = torch.device(device)
-        f32 = dict(dtype=torch.float32, device=self.device)
-        self.x = torch.empty(n, self.ld, **f32)
-        self.mu = torch.empty(n, self.ld, **f32)
-        self.msg = [torch.empty(max(self.E, 1), self.ld, **f32) for _ in range(2)]
-        self.counts = torch.zeros(max(self.E, 1), dtype=torch.int32, device=self.device)
-        self.t = 0
-        self.cur = 0  # msg[cur] holds m^{t-1}
-
-    def init(self, x0_std: float, seed: int, mix, mu_scale: float, mu_seed: int, sigma: float):
-        import torch
-        mix_t = torch.as_tensor(np.asarray(mix, dtype=np.float32), device=self.device).contiguous()
-        relay_fill_objective(self.h, self.mu, mix_t, mix_t.shape[1], mu_scale, mu_seed)
-        relay_set_objective(self.h, self.mu, sigma)
-        relay_init(self.h, self.x, self.msg[0], self.msg[1], self.counts, x0_std, seed)
-        self._mix = mix_t  # keep alive until the fill has run
-        self.t = 0
-        self.cur = 0
-
-    def step(self, lr: float, seed: int, stream=None):
-        relay_step(self.h, self.x, self.msg[self.cur], self.msg[1 - self.cur], self.counts, lr,
-                   seed, self.t, stream)
-        self.cur = 1 - self.cur
-        self.t += 1
+    def __init__(self, h, col0: int, d: int, E: int, msg, counts):
+        self.h, self.col0, self.d, self.E = h, col0, d, E
+        self.msg = msg          # two [E][ld_msg] buffers (double buffering)
+        self.counts = counts    # int32 [E]
+        self.cur = 0            # msg[cur] holds m^{t-1}
 
     @property
     def messages(self):
-        """m^{t-1}: the messages of the last step."""
         return self.msg[self.cur]
+
+
+def _window_ptr(t, col0: int) -> int:
+    return t.data_ptr() + 4 * col0
+
+
+class RelayRun:
+    """Device state of one RelaySGD run, allocated with torch on `device`.
+
+    `edges` is one tree, or a list of trees that split the coordinates into
+    contiguous quad-aligned windows of the same model array -- the double
+    binary trees of Section 3 are a list of two.  Buffers: x [n][ld], per tree
+    two message buffers [E][ld_tree] (double buffering) and counters int32
+    [E], and -- for objective="stored" -- the centres mu [n][ld]
+    (objective="generated" lets the kernel regenerate them).  ``step()``
+    enqueues one relay_step per tree on the current torch stream.
+    """
+
+    def __init__(self, n: int, d: int, edges, device="cuda", mode: int = 1, c0: int = 0,
+                 objective: str = "stored"):
+        import torch
+        if objective not in ("stored", "generated"):
+            raise ValueError(objective)
+        trees = list(edges) if isinstance(edges, (list, tuple)) else [edges]
+        self.objective = objective
+        self.n, self.d, self.c0 = n, d, c0
+        self.device = torch.device(device)
+        self.ld = (d + 31) // 32 * 32
+        f32 = dict(dtype=torch.float32, device=self.device)
+        self.x = torch.empty(n, self.ld, **f32)
+        self.mu = torch.empty(n, self.ld, **f32) if objective == "stored" else None
+        nq = (d + 3) // 4
+        self.trees = []
+        for k, tree_edges in enumerate(trees):
+            q_lo, q_hi = nq * k // len(trees), nq * (k + 1) // len(trees)
+            col0 = 4 * q_lo
+            dk = min(4 * q_hi, d) - col0 if q_hi > q_lo else 0
+            h = relay_create(n, dk, tree_edges)
+            relay_set_rebuild_mode(h, mode)
+            relay_set_coord_offset(h, c0 + col0)
+            ld_m = relay_ld(h)
+            relay_set_strides(h, self.ld, ld_m)
+            E = relay_num_edges(h)
+            msg = [torch.empty(max(E, 1), max(ld_m, 1), **f32) for _ in range(2)]
+            counts = torch.zeros(max(E, 1), dtype=torch.int32, device=self.device)
+            self.trees.append(_TreeState(h, col0, dk, E, msg, counts))
+        self.t = 0
+
+    # single-tree conveniences
+    @property
+    def h(self):
+        return self.trees[0].h
+
+    @property
+    def E(self) -> int:
+        return self.trees[0].E
+
+    @property
+    def counts(self):
+        return self.trees[0].counts
+
+    @property
+    def msg(self):
+        return self.trees[0].msg
+
+    @property
+    def cur(self) -> int:
+        return self.trees[0].cur
+
+    @cur.setter
+    def cur(self, v: int):
+        self.trees[0].cur = v
+
+    @property
+    def messages(self):
+        """m^{t-1} of the first tree: the messages of the last step."""
+        return self.trees[0].messages
+
+    def _x(self, tr):
+        return _window_ptr(self.x, tr.col0) if tr.d > 0 else None
+
+    def init(self, x0_std: float, seed: int, mix, mu_scale: float, mu_seed: int, sigma: float):
+        import torch
+        mix = np.asarray(mix, dtype=np.float32)
+        mix_t = None
+        for tr in self.trees:
+            if self.objective == "stored":
+                if mix_t is None:
+                    mix_t = torch.as_tensor(mix, device=self.device).contiguous()
+                mu = _window_ptr(self.mu, tr.col0) if tr.d > 0 else None
+                relay_fill_objective(tr.h, mu, mix_t, mix_t.shape[1], mu_scale, mu_seed)
+                relay_set_objective(tr.h, mu, sigma)
+            else:
+                relay_set_objective_generated(tr.h, mix, mix.shape[1], mu_scale, mu_seed, sigma)
+            relay_init(tr.h, self._x(tr), tr.msg[0], tr.msg[1], tr.counts, x0_std, seed)
+            tr.cur = 0
+        self._mix = mix_t  # keep alive until the fills have run
+        self.t = 0
+
+    def step(self, lr: float, seed: int, stream=None):
+        for tr in self.trees:
+            relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed,
+                       self.t, stream)
+            tr.cur = 1 - tr.cur
+        self.t += 1

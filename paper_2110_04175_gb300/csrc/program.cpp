@@ -120,10 +120,16 @@ Walk make_walk(const Tree& t, int root) {
         std::stable_sort(ch.begin(), ch.end(), [&](int a, int b) { return need[a] > need[b]; });
         const int m = static_cast<int>(ch.size());
         const int D = static_cast<int>(t.nbr[i].size());
+        // slots held by i while its children's subtrees are walked:
+        // narrow: accumulator + one pending message per later child;
+        // wide: accumulator + total (children read the total, no pending messages)
+        const bool wide = D > kRegDeg;
         int peak = (w.parent[i] >= 0) ? 1 : 0;
-        peak = std::max(peak, (m > 0 ? 1 : 0) + (D > kRegDeg ? D : m));
-        for (int k = 0; k < m; ++k) peak = std::max(peak, (m > 0 ? 1 : 0) + (m - 1 - k) + need[ch[k]]);
-        need[i] = peak;
+        const int own = (m > 0) ? (wide ? 2 : 1) : 0;
+        peak = std::max(peak, own + (wide ? 0 : m));
+        for (int k = 0; k < m; ++k)
+            peak = std::max(peak, own + (wide ? 0 : (m - 1 - k)) + need[ch[k]] - (wide ? 1 : 0));
+        need[i] = std::max(peak, 1);
     }
     // pre-order
     std::vector<int> stack{root};
@@ -154,7 +160,7 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
     auto release = [&](int s) {
         if (s >= 0) free_ids.push(s);
     };
-    std::vector<int> recv(n, -1), acc(n, -1), pos_base(n, 0);
+    std::vector<int> recv(n, -1), acc(n, -1), tot(n, -1), pos_base(n, 0);
     int base = 0;
     for (int i = 0; i < n; ++i) {
         pos_base[i] = base;
@@ -165,8 +171,13 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
         const int par = w.parent[i];
         const int D = static_cast<int>(t.nbr[i].size());
         const int m = static_cast<int>(w.children[i].size());
-        release(recv[i]);  // read first, at the start of the visit
+        const bool wide = D > kRegDeg;
+        const bool par_wide = par >= 0 && static_cast<int>(t.nbr[par].size()) > kRegDeg;
+        // a message slot is read at the start of the visit and freed; a
+        // wide parent's total stays live until its last child
+        if (!par_wide) release(recv[i]);
         acc[i] = (m > 0) ? alloc() : -1;
+        tot[i] = (wide && m > 0) ? alloc() : -1;
         int parent_pos = -1;
         for (int s = 0; s < D; ++s) {
             const int k = t.nbr[i][s];
@@ -175,9 +186,15 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
             p->pos_out[pos] = static_cast<int16_t>(t.out_edge[i][s]);
             if (k == par) parent_pos = s;
             int slot = -1;
-            if (D > kRegDeg || k != par) slot = alloc();
+            if (k != par) {
+                if (wide) {
+                    recv[k] = tot[i];
+                } else {
+                    slot = alloc();
+                    recv[k] = slot;
+                }
+            }
             p->pos_slot[pos] = static_cast<int16_t>(slot);
-            if (k != par) recv[k] = slot;
         }
         NodeRec& r = p->node[i];
         r.deg = static_cast<int16_t>(D);
@@ -189,8 +206,12 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
         const bool last = par >= 0 && w.children[par].back() == i;
         r.fin_parent = static_cast<int16_t>(last ? par : -1);
         r.parent = static_cast<int16_t>(par);
-        if (D > kRegDeg && parent_pos >= 0) release(p->pos_slot[pos_base[i] + parent_pos]);
-        if (last) release(acc[par]);
+        r.tot_slot = static_cast<int16_t>(tot[i]);
+        r.flags = static_cast<int16_t>(par_wide ? kRecvFromTotal : 0);
+        if (last) {
+            release(acc[par]);
+            release(tot[par]);
+        }
         p->order[v] = static_cast<int16_t>(i);
     }
     (void)root;

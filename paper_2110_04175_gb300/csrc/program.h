@@ -4,12 +4,22 @@
 // thread owns a quad of coordinates for ALL workers and walks the tree once
 // per step.  The walk is a depth-first pre-order from a chosen root.  At the
 // visit of worker i the thread forms x_i^{t+1/2}, reads the D = |N(i)|
-// incoming messages m^{t-1}_{k->i}, writes the D outgoing messages
+// incoming messages m^{t-1}_{k->i} and produces the D outgoing messages
 // m^t_{i->k} (each the sum of x_i^{t+1/2} and the OTHER D-1 incoming
-// messages), and routes them into the rebuild sums: the message to the DFS
+// messages), routing them into the rebuild sums: the message to the DFS
 // parent goes straight into the parent's accumulator, a message to a child
 // waits in a shared-memory slot until that child is visited.  A worker's
 // rebuild finishes at the visit of its last child (or its own, for a leaf).
+//
+// Two ways to form the outgoing messages:
+//   - degree <= kRegDeg ("narrow"): the incoming messages stay in registers
+//     and message s is a prefix sum plus a suffix sum over the others;
+//   - degree > kRegDeg ("wide", e.g. a star's hub): one streaming pass forms
+//     the total T_i = x_i^{t+1/2} + sum_k m^{t-1}_{k->i}; only T_i is kept
+//     (one slot), and each child c forms its own incoming message as
+//     m^t_{i->c} = T_i - m^{t-1}_{c->i} at its visit (re-reading that one
+//     message) and writes it out.  This keeps the slots per thread O(1)
+//     instead of O(degree).
 //
 // The program is a plain-old-data struct passed by value as a
 // __grid_constant__ kernel parameter (warp-uniform reads from the constant
@@ -24,15 +34,21 @@ constexpr int kMaxN = 256;               // == RELAY_MAX_N
 constexpr int kMaxE = 2 * (kMaxN - 1);
 constexpr int kRegDeg = 4;               // degrees up to this keep messages in registers
 
-struct NodeRec {        // 16 bytes; indexed by worker id
+enum NodeFlags : int16_t {
+    kRecvFromTotal = 1,  // recv_slot holds the wide parent's total T_p
+};
+
+struct NodeRec {        // 20 bytes; indexed by worker id
     int16_t deg;        // D = |N(i)|
     int16_t pos_base;   // first of i's D positions (ascending neighbour id)
     int16_t parent_pos; // position of the DFS parent among i's neighbours; -1 at the root
-    int16_t recv_slot;  // slot holding m^t_{parent->i}; -1 at the root
+    int16_t recv_slot;  // slot holding m^t_{parent->i} (or T_parent); -1 at the root
     int16_t acc_slot;   // slot of i's rebuild accumulator; -1 for a leaf
     int16_t parent_acc; // the parent's accumulator slot; -1 at the root
     int16_t fin_parent; // parent id when i is the parent's last child, else -1
     int16_t parent;     // DFS parent id; -1 at the root
+    int16_t tot_slot;   // wide node with children: slot of its total T_i; else -1
+    int16_t flags;      // NodeFlags
 };
 
 struct Program {
@@ -41,10 +57,29 @@ struct Program {
     NodeRec node[kMaxN];
     int16_t pos_in[kMaxE];       // position s of i: edge k_s -> i
     int16_t pos_out[kMaxE];      // position s of i: edge i -> k_s
-    int16_t pos_slot[kMaxE];     // slot of the message to child k_s (every
-                                 // position when D > kRegDeg: suffix-sum scratch)
+    int16_t pos_slot[kMaxE];     // narrow node: slot of the message to child k_s; else -1
     int16_t edge_src[kMaxE];     // directed edge e: edge_src[e] -> edge_dst[e]
     int16_t edge_dst[kMaxE];
+};
+
+// Where the kernel takes the quadratic centres mu_i from.
+constexpr int kMaxMixNnz = 1024;        // non-zero mixture weights in a kernel parameter
+constexpr int kMaxCachedCentres = 16;   // centres kept per thread in shared memory
+
+enum ObjectiveSource : int32_t {
+    kMuStored = 0,      // read the caller's mu array
+    kMuPerRow = 1,      // regenerate: one Philox block per non-zero weight of the row
+    kMuCachedCentres = 2,  // regenerate the K centres once per quad, then mix per row
+};
+
+struct Objective {
+    int32_t source;     // ObjectiveSource
+    int32_t K;          // centres
+    float scale;        // mu_i = scale * sum_k w_ik N_k
+    uint32_t k0, k1;    // Philox key of the centres (stream 1)
+    int16_t row_off[kMaxN + 1];   // row i's non-zeros: [row_off[i], row_off[i+1])
+    int16_t col[kMaxMixNnz];      // centre index, ascending within a row
+    float w[kMaxMixNnz];          // weight
 };
 
 // Status codes mirror relaysum.h.

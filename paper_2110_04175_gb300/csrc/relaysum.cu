@@ -11,9 +11,9 @@
 //                         local step with Philox noise, every outgoing relay
 //                         message, every rebuild.  Each x_i, mu_i and incoming
 //                         message quad is read from HBM once and each outgoing
-//                         message / new model quad written once (the generic
-//                         path for degree > 4 re-reads its incoming messages
-//                         once more, from cache).  The path is bandwidth-bound
+//                         message / new model quad written once (a child of a
+//                         node of degree > 4 re-reads the one message it sent
+//                         that node, see program.h).  The path is bandwidth-bound
 //                         streaming arithmetic: no tensor cores.
 //   relay_init_kernel     x^0 (shared Philox draw) and zeroed messages.
 //   relay_fill_mu_kernel  mu_i = scale * sum_k mix[i][k] N_k.
@@ -32,11 +32,14 @@ using relaysum::kMaxE;
 using relaysum::kMaxN;
 using relaysum::kRegDeg;
 using relaysum::NodeRec;
+using relaysum::Objective;
 using relaysum::Program;
 
 struct relay_handle {
     Program prog;
+    Objective obj;
     int64_t d = 0, ld = 0, nquads = 0, c0 = 0;
+    int64_t ld_x = 0, ld_m = 0;  // row strides (floats) of x / mu and of the messages
     int32_t mode = 1;
     const float* mu = nullptr;
     float sigma = 0.0f;
@@ -54,14 +57,29 @@ constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;
 constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;
 constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
 
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+// The ten round keys (k0 + r W0, k1 + r W1), computed once on the host.
+struct PhiloxKey {
+    uint32_t k[10][2];
+};
+
+PhiloxKey philox_key(uint64_t seed) {
+    PhiloxKey key;
+    uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
+    for (int r = 0; r < 10; ++r) {
+        key.k[r][0] = k0;
+        key.k[r][1] = k1;
+        k0 += kPhiloxW0;
+        k1 += kPhiloxW1;
+    }
+    return key;
+}
+
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, const PhiloxKey& key) {
 #pragma unroll
     for (int round = 0; round < 10; ++round) {
         const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
         const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
-        c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
-        k0 += kPhiloxW0;
-        k1 += kPhiloxW1;
+        c = make_uint4(hi1 ^ c.y ^ key.k[round][0], lo1, hi0 ^ c.w ^ key.k[round][1], lo0);
     }
     return c;
 }
@@ -71,17 +89,28 @@ __device__ __forceinline__ float unit_interval(uint32_t w) {
     return __uint2float_rn((w >> 8) + 1u) * 5.9604644775390625e-8f;  // 2^-24
 }
 
+__device__ __forceinline__ float sqrt_approx(float v) {
+    float r;
+    asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(v));
+    return r;
+}
+
 // Four standard normals for coordinates 4q .. 4q+3 (Box-Muller on the two
-// word pairs of one Philox block).
+// word pairs of one Philox block): z = sqrt(-2 ln u_a) (cos, sin)(2 pi u_b).
+// The angle is taken as 2 pi u_b - pi, inside the range where the hardware
+// sine/cosine are accurate to 2^-21.4, and the half turn is undone by the
+// sign; the radius keeps an accurate logarithm (its argument can sit just
+// below 1, where an approximate one loses all relative accuracy).
 __device__ __forceinline__ float4 normal4(uint32_t q, uint32_t row, uint32_t step, uint32_t stream,
-                                          uint32_t k0, uint32_t k1) {
-    const uint4 w = philox4x32_10(make_uint4(q, row, step, stream), k0, k1);
-    const float r0 = sqrtf(-2.0f * logf(unit_interval(w.x)));
-    const float r1 = sqrtf(-2.0f * logf(unit_interval(w.z)));
+                                          const PhiloxKey& key) {
+    const uint4 w = philox4x32_10(make_uint4(q, row, step, stream), key);
+    const float r0 = sqrt_approx(-2.0f * logf(unit_interval(w.x)));
+    const float r1 = sqrt_approx(-2.0f * logf(unit_interval(w.z)));
+    constexpr float kTwoPi = 6.28318530717958647692f, kPi = 3.14159265358979323846f;
     float s0, c0, s1, c1;
-    sincospif(2.0f * unit_interval(w.y), &s0, &c0);
-    sincospif(2.0f * unit_interval(w.w), &s1, &c1);
-    return make_float4(r0 * c0, r0 * s0, r1 * c1, r1 * s1);
+    __sincosf(fmaf(unit_interval(w.y), kTwoPi, -kPi), &s0, &c0);
+    __sincosf(fmaf(unit_interval(w.w), kTwoPi, -kPi), &s1, &c1);
+    return make_float4(-r0 * c0, -r0 * s0, -r1 * c1, -r1 * s1);
 }
 
 // ------------------------------------------------------------ float4 helpers
@@ -89,11 +118,35 @@ __device__ __forceinline__ float4 normal4(uint32_t q, uint32_t row, uint32_t ste
 __device__ __forceinline__ float4 add4(float4 a, float4 b) {
     return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
+__device__ __forceinline__ float4 sub4(float4 a, float4 b) {
+    return make_float4(a.x - b.x, a.y - b.y, a.z - b.z, a.w - b.w);
+}
 __device__ __forceinline__ float4 scale4(float4 a, float s) {
     return make_float4(a.x * s, a.y * s, a.z * s, a.w * s);
 }
+// Rounded product that the compiler may not fuse into a later add: the
+// regenerated mu must round exactly like the stored one.
+__device__ __forceinline__ float4 scale4_rn(float4 a, float s) {
+    return make_float4(__fmul_rn(a.x, s), __fmul_rn(a.y, s), __fmul_rn(a.z, s), __fmul_rn(a.w, s));
+}
+__device__ __forceinline__ float4 fma4(float w, float4 z, float4 acc) {
+    return make_float4(fmaf(w, z.x, acc.x), fmaf(w, z.y, acc.y), fmaf(w, z.z, acc.z), fmaf(w, z.w, acc.w));
+}
+// Loads read once per step stream through L2 with evict-first priority.
 __device__ __forceinline__ float4 ld_stream(const float* p) {
-    return __ldg(reinterpret_cast<const float4*>(p));
+    return __ldcs(reinterpret_cast<const float4*>(p));
+}
+// A wide node's incoming messages are read again at its children's visits
+// (program.h): keep them in L2 with evict-last priority until then.
+__device__ __forceinline__ float4 ld_keep(const float* p) {
+    float4 v;
+    asm volatile(
+        "{\n\t.reg .b64 pol;\n\t"
+        "createpolicy.fractional.L2::evict_last.b64 pol, 1.0;\n\t"
+        "ld.global.nc.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], pol;\n\t}"
+        : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+        : "l"(p));
+    return v;
 }
 __device__ __forceinline__ void st_stream(float* p, float4 v) {
     __stcs(reinterpret_cast<float4*>(p), v);
@@ -127,12 +180,13 @@ struct ModelArgs {
     const float* msg_in;
     float* msg_out;
     const int32_t* counts;
-    int64_t ld;       // row stride (floats)
+    int64_t ld_x;     // row stride (floats) of x and mu
+    int64_t ld_m;     // row stride (floats) of the messages
     int64_t nquads;   // ceil(d / 4)
     uint32_t q0;      // absolute quad of local coordinate 0
     uint32_t step;
-    uint32_t k0, k1;  // Philox key
     float lr, sigma;
+    PhiloxKey key;    // noise key schedule
 };
 
 // Per-thread view of the shared-memory slots: slot s of this thread is
@@ -149,7 +203,7 @@ __device__ __forceinline__ void to_parent(const NodeRec& r, const ModelArgs& a, 
                                           const Slots& sl, const float* s_scale) {
     const float4 acc = add4(sl[r.parent_acc], out);
     if (r.fin_parent >= 0) {
-        st_stream(a.x + r.fin_parent * a.ld + 4 * q, scale4(acc, s_scale[r.fin_parent]));
+        st_stream(a.x + r.fin_parent * a.ld_x + 4 * q, scale4(acc, s_scale[r.fin_parent]));
     } else {
         sl[r.parent_acc] = acc;
     }
@@ -163,7 +217,7 @@ __device__ __forceinline__ void visit_small(const Program& prog, const NodeRec& 
                                             const float* s_scale) {
     float4 m[D];
 #pragma unroll
-    for (int s = 0; s < D; ++s) m[s] = ld_stream(a.msg_in + prog.pos_in[r.pos_base + s] * a.ld + 4 * q);
+    for (int s = 0; s < D; ++s) m[s] = ld_stream(a.msg_in + prog.pos_in[r.pos_base + s] * a.ld_m + 4 * q);
     float4 pre[D];
     pre[0] = xh;
 #pragma unroll
@@ -175,7 +229,7 @@ __device__ __forceinline__ void visit_small(const Program& prog, const NodeRec& 
 #pragma unroll
     for (int s = 0; s < D; ++s) {
         const float4 out = (s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]);
-        st_stream(a.msg_out + prog.pos_out[r.pos_base + s] * a.ld + 4 * q, out);
+        st_stream(a.msg_out + prog.pos_out[r.pos_base + s] * a.ld_m + 4 * q, out);
         if (s == r.parent_pos) {
             to_parent(r, a, q, out, sl, s_scale);
         } else {
@@ -184,38 +238,53 @@ __device__ __forceinline__ void visit_small(const Program& prog, const NodeRec& 
     }
 }
 
-// Degree D > kRegDeg: suffix sums go to the node's position slots on a
-// descending pass; an ascending pass re-reads each incoming message (from
-// cache) to extend the prefix and overwrites slot s with message s.
-__device__ __noinline__ void visit_generic(const Program& prog, const NodeRec& r, const ModelArgs& a,
-                                           int64_t q, float4 xh, const Slots& sl,
-                                           const float* s_scale) {
+// Degree D > kRegDeg: one streaming pass forms T = xh + sum of all incoming
+// messages; the message to the parent is T minus the parent's incoming
+// message, and T stays in a slot for the children (see program.h).
+__device__ __noinline__ void visit_wide(const Program& prog, const NodeRec& r, const ModelArgs& a,
+                                        int64_t q, float4 xh, const Slots& sl,
+                                        const float* s_scale) {
     const int D = r.deg;
     const int base = r.pos_base;
-    float4 suf = ld_stream(a.msg_in + prog.pos_in[base + D - 1] * a.ld + 4 * q);
-    sl[prog.pos_slot[base + D - 1]] = suf;
-    for (int s = D - 2; s >= 0; --s) {
-        suf = add4(ld_stream(a.msg_in + prog.pos_in[base + s] * a.ld + 4 * q), suf);
-        sl[prog.pos_slot[base + s]] = suf;
-    }
-    float4 pre = xh;
+    float4 total = xh;
+    float4 from_parent = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int s = 0; s < D; ++s) {
-        const float4 out = (s == D - 1) ? pre : add4(pre, sl[prog.pos_slot[base + s + 1]]);
-        pre = add4(pre, ld_stream(a.msg_in + prog.pos_in[base + s] * a.ld + 4 * q));
-        st_stream(a.msg_out + prog.pos_out[base + s] * a.ld + 4 * q, out);
-        if (s == r.parent_pos) {
-            to_parent(r, a, q, out, sl, s_scale);
-        } else {
-            sl[prog.pos_slot[base + s]] = out;
-        }
+        const float4 m = ld_keep(a.msg_in + prog.pos_in[base + s] * a.ld_m + 4 * q);
+        total = add4(total, m);
+        if (s == r.parent_pos) from_parent = m;
     }
+    if (r.parent_pos >= 0) {
+        const float4 out = sub4(total, from_parent);
+        st_stream(a.msg_out + prog.pos_out[base + r.parent_pos] * a.ld_m + 4 * q, out);
+        to_parent(r, a, q, out, sl, s_scale);
+    }
+    sl[r.tot_slot] = total;
+}
+
+// mu_i for quad q: read, or regenerated exactly as relay_fill_mu_kernel
+// writes it (same normals, same fma order), so both sources give the same bits.
+template <int OBJ>
+__device__ __forceinline__ float4 centre(const Objective& obj, const PhiloxKey& mu_key, const ModelArgs& a,
+                                         int i, int64_t q, const float4* cen, int cen_stride) {
+    if (OBJ == relaysum::kMuStored) return ld_stream(a.mu + i * a.ld_x + 4 * q);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int j = obj.row_off[i]; j < obj.row_off[i + 1]; ++j) {
+        const float4 z = (OBJ == relaysum::kMuPerRow)
+                             ? normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(obj.col[j]),
+                                       0u, 1u, mu_key)
+                             : cen[obj.col[j] * cen_stride];
+        acc = fma4(obj.w[j], z, acc);
+    }
+    return scale4_rn(acc, obj.scale);
 }
 
 // MODE 0: x' = acc / nbar (Alg. 1).  MODE 1: x' = (acc + (n - nbar) x) / n
 // (robust rule), with the fill term folded into the accumulator up front.
-template <int MODE>
+// OBJ: where mu comes from (ObjectiveSource).
+template <int MODE, int OBJ>
 __global__ void __launch_bounds__(128)
-relay_models_kernel(const __grid_constant__ Program prog, const ModelArgs a) {
+relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant__ Objective obj,
+                    const __grid_constant__ PhiloxKey mu_key, const __grid_constant__ ModelArgs a) {
     extern __shared__ float4 slot_mem[];
     __shared__ float s_scale[kMaxN];
     __shared__ float s_fill[kMaxN];
@@ -234,16 +303,22 @@ relay_models_kernel(const __grid_constant__ Program prog, const ModelArgs a) {
     }
     __syncthreads();
     const Slots sl{slot_mem + threadIdx.x, static_cast<int>(blockDim.x)};
+    float4* cen = slot_mem + prog.nslots * blockDim.x + threadIdx.x;  // OBJ == kMuCachedCentres
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
     for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < a.nquads;
          q += stride) {
+        if (OBJ == relaysum::kMuCachedCentres) {
+            for (int k = 0; k < obj.K; ++k)
+                cen[k * blockDim.x] = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k), 0u,
+                                              1u, mu_key);
+        }
         for (int v = 0; v < n; ++v) {
             const int i = prog.order[v];
             const NodeRec r = prog.node[i];
-            const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld + 4 * q);
-            const float4 mv = ld_stream(a.mu + i * a.ld + 4 * q);
+            const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
+            const float4 mv = centre<OBJ>(obj, mu_key, a, i, q, cen, static_cast<int>(blockDim.x));
             const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i),
-                                     a.step, 0u, a.k0, a.k1);
+                                     a.step, 0u, a.key);
             // x^{t+1/2} = x - lr * ((x - mu) + sigma * xi)
             float4 xh;
             xh.x = fmaf(-a.lr, fmaf(a.sigma, z.x, xv.x - mv.x), xv.x);
@@ -252,17 +327,26 @@ relay_models_kernel(const __grid_constant__ Program prog, const ModelArgs a) {
             xh.w = fmaf(-a.lr, fmaf(a.sigma, z.w, xv.w - mv.w), xv.w);
             float4 acc = xh;
             if (MODE == 1) acc = add4(scale4(xv, s_fill[i]), xh);
-            if (r.recv_slot >= 0) acc = add4(acc, sl[r.recv_slot]);
+            if (r.recv_slot >= 0) {
+                float4 recv = sl[r.recv_slot];
+                if (r.flags & relaysum::kRecvFromTotal) {
+                    // m^t_{p->i} = T_p - m^{t-1}_{i->p}, written out here
+                    const int pos = r.pos_base + r.parent_pos;
+                    recv = sub4(recv, ld_stream(a.msg_in + prog.pos_out[pos] * a.ld_m + 4 * q));
+                    st_stream(a.msg_out + prog.pos_in[pos] * a.ld_m + 4 * q, recv);
+                }
+                acc = add4(acc, recv);
+            }
             switch (r.deg) {
                 case 0: break;
                 case 1: visit_small<1>(prog, r, a, q, xh, sl, s_scale); break;
                 case 2: visit_small<2>(prog, r, a, q, xh, sl, s_scale); break;
                 case 3: visit_small<3>(prog, r, a, q, xh, sl, s_scale); break;
                 case 4: visit_small<4>(prog, r, a, q, xh, sl, s_scale); break;
-                default: visit_generic(prog, r, a, q, xh, sl, s_scale); break;
+                default: visit_wide(prog, r, a, q, xh, sl, s_scale); break;
             }
             if (r.acc_slot < 0) {
-                st_stream(a.x + i * a.ld + 4 * q, scale4(acc, s_scale[i]));
+                st_stream(a.x + i * a.ld_x + 4 * q, scale4(acc, s_scale[i]));
             } else {
                 sl[r.acc_slot] = acc;
             }
@@ -272,49 +356,41 @@ relay_models_kernel(const __grid_constant__ Program prog, const ModelArgs a) {
 
 // --------------------------------------------------------------------- init
 
-__global__ void relay_init_kernel(float* x, float* msg_a, float* msg_b, int n, int E, int64_t ld,
-                                  int64_t d, uint32_t q0, float x0_std, uint32_t k0, uint32_t k1) {
-    const int64_t ld4 = ld / 4;
+__global__ void relay_init_kernel(float* x, float* msg_a, float* msg_b, int n, int E, int64_t ld_x,
+                                  int64_t ld_m, int64_t nquads, int64_t d, uint32_t q0, float x0_std,
+                                  const __grid_constant__ PhiloxKey key) {
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < ld4; q += stride) {
-        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < nquads; q += stride) {
         const int64_t c = 4 * q;
-        if (c < d) {
-            const float4 z = normal4(q0 + static_cast<uint32_t>(q), 0u, 0u, 2u, k0, k1);
-            v = make_float4(x0_std * z.x, c + 1 < d ? x0_std * z.y : 0.f,
-                            c + 2 < d ? x0_std * z.z : 0.f, c + 3 < d ? x0_std * z.w : 0.f);
-        }
-        for (int i = 0; i < n; ++i) reinterpret_cast<float4*>(x)[i * ld4 + q] = v;
+        const float4 z = normal4(q0 + static_cast<uint32_t>(q), 0u, 0u, 2u, key);
+        const float4 v = make_float4(x0_std * z.x, c + 1 < d ? x0_std * z.y : 0.f,
+                                     c + 2 < d ? x0_std * z.z : 0.f, c + 3 < d ? x0_std * z.w : 0.f);
+        for (int i = 0; i < n; ++i) *reinterpret_cast<float4*>(x + i * ld_x + c) = v;
         const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int e = 0; e < E; ++e) {
-            reinterpret_cast<float4*>(msg_a)[e * ld4 + q] = zero;
-            if (msg_b) reinterpret_cast<float4*>(msg_b)[e * ld4 + q] = zero;
+            *reinterpret_cast<float4*>(msg_a + e * ld_m + c) = zero;
+            if (msg_b) *reinterpret_cast<float4*>(msg_b + e * ld_m + c) = zero;
         }
     }
 }
 
-__global__ void relay_fill_mu_kernel(float* mu, const float* mix, int n, int K, int64_t ld, int64_t d,
-                                     uint32_t q0, float scale, uint32_t k0, uint32_t k1) {
-    const int64_t ld4 = ld / 4;
+__global__ void relay_fill_mu_kernel(float* mu, const float* mix, int n, int K, int64_t ld_x, int64_t nquads,
+                                     int64_t d, uint32_t q0, float scale, const __grid_constant__ PhiloxKey key) {
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < ld4; q += stride) {
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < nquads; q += stride) {
         const int64_t c = 4 * q;
         for (int i = 0; i < n; ++i) {
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (c < d) {
-                for (int k = 0; k < K; ++k) {
-                    const float w = __ldg(mix + static_cast<int64_t>(i) * K + k);
-                    if (w != 0.0f) {  // a zero weight adds exactly nothing
-                        const float4 z = normal4(q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k),
-                                                 0u, 1u, k0, k1);
-                        acc = make_float4(fmaf(w, z.x, acc.x), fmaf(w, z.y, acc.y),
-                                          fmaf(w, z.z, acc.z), fmaf(w, z.w, acc.w));
-                    }
+            for (int k = 0; k < K; ++k) {
+                const float w = __ldg(mix + static_cast<int64_t>(i) * K + k);
+                if (w != 0.0f) {  // a zero weight adds exactly nothing
+                    const float4 z = normal4(q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k), 0u, 1u, key);
+                    acc = fma4(w, z, acc);
                 }
             }
-            const float4 v = make_float4(scale * acc.x, c + 1 < d ? scale * acc.y : 0.f,
-                                         c + 2 < d ? scale * acc.z : 0.f, c + 3 < d ? scale * acc.w : 0.f);
-            reinterpret_cast<float4*>(mu)[i * ld4 + q] = c < d ? v : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 sv = scale4_rn(acc, scale);
+            *reinterpret_cast<float4*>(mu + i * ld_x + c) =
+                make_float4(sv.x, c + 1 < d ? sv.y : 0.f, c + 2 < d ? sv.z : 0.f, c + 3 < d ? sv.w : 0.f);
         }
     }
 }
@@ -358,31 +434,42 @@ int models_threads(int nslots) {
     return t;
 }
 
-template <int MODE>
+template <int MODE, int OBJ>
 int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
     int dev = 0;
     const int sms = device_sms(&dev);
     if (sms <= 0) return RELAY_ECUDA;
-    const int threads = models_threads(h->prog.nslots);
-    const size_t smem = static_cast<size_t>(h->prog.nslots) * threads * 16;
+    const int per_thread = h->prog.nslots + (OBJ == relaysum::kMuCachedCentres ? h->obj.K : 0);
+    const int threads = models_threads(per_thread);
+    const size_t smem = static_cast<size_t>(per_thread) * threads * 16;
     if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
     static std::atomic<bool> smem_set[kMaxDevices];
     if (smem > 48 * 1024 && dev < kMaxDevices && !smem_set[dev].load()) {
-        if (cudaFuncSetAttribute(relay_models_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(relay_models_kernel<MODE, OBJ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kMaxSmem) != cudaSuccess)
             return RELAY_ECUDA;
         smem_set[dev].store(true);
     }
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_models_kernel<MODE>, threads, smem) !=
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_models_kernel<MODE, OBJ>, threads, smem) !=
             cudaSuccess ||
         per_sm <= 0)
         return RELAY_ECUDA;
     const int64_t want = (a.nquads + threads - 1) / threads;
     const int64_t cap = static_cast<int64_t>(sms) * per_sm;
     const int grid = static_cast<int>(want < cap ? want : cap);
-    relay_models_kernel<MODE><<<grid, threads, smem, stream>>>(h->prog, a);
+    const PhiloxKey mu_key = philox_key(static_cast<uint64_t>(h->obj.k0) | (static_cast<uint64_t>(h->obj.k1) << 32));
+    relay_models_kernel<MODE, OBJ><<<grid, threads, smem, stream>>>(h->prog, h->obj, mu_key, a);
     return launch_status();
+}
+
+template <int MODE>
+int launch_models_obj(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
+    switch (h->obj.source) {
+        case relaysum::kMuStored: return launch_models<MODE, relaysum::kMuStored>(h, a, stream);
+        case relaysum::kMuPerRow: return launch_models<MODE, relaysum::kMuPerRow>(h, a, stream);
+        default: return launch_models<MODE, relaysum::kMuCachedCentres>(h, a, stream);
+    }
 }
 
 // Argument checks shared by relay_step_models and relay_step.
@@ -396,7 +483,9 @@ int check_step_args(const relay_handle* h, const float* x, const float* msg_in, 
     if (E > 0 && (!msg_in || !msg_out || msg_in == msg_out)) return RELAY_EINVAL;
     if (!x || !aligned16(x) || (E > 0 && (!aligned16(msg_in) || !aligned16(msg_out))))
         return RELAY_EINVAL;
-    const int64_t xb = h->prog.n * h->ld * 4, mb = E * h->ld * 4;
+    // exact byte spans of the strided arrays (windows of wider arrays may sit side by side)
+    const int64_t xb = ((h->prog.n - 1) * h->ld_x + 4 * h->nquads) * 4;
+    const int64_t mb = E > 0 ? ((E - 1) * h->ld_m + 4 * h->nquads) * 4 : 0;
     if (overlap(x, xb, msg_in, mb) || overlap(x, xb, msg_out, mb) || overlap(msg_in, mb, msg_out, mb))
         return RELAY_EINVAL;
     return RELAY_OK;
@@ -436,6 +525,8 @@ int relay_create(relay_handle** out, int32_t n, int64_t d, const int32_t* edges,
     }
     h->d = d;
     h->ld = ld;
+    h->ld_x = ld;
+    h->ld_m = ld;
     h->nquads = (d + 3) / 4;
     *out = h;
     return RELAY_OK;
@@ -453,6 +544,13 @@ int relay_edges(const relay_handle* h, int32_t* src, int32_t* dst) {
         src[e] = h->prog.edge_src[e];
         dst[e] = h->prog.edge_dst[e];
     }
+    return RELAY_OK;
+}
+
+int relay_set_strides(relay_handle* h, int64_t ld_x, int64_t ld_msg) {
+    if (!h || ld_x < 4 * h->nquads || ld_msg < 4 * h->nquads || (ld_x & 3) || (ld_msg & 3)) return RELAY_EINVAL;
+    h->ld_x = ld_x;
+    h->ld_m = ld_msg;
     return RELAY_OK;
 }
 
@@ -474,6 +572,44 @@ int relay_set_objective(relay_handle* h, const float* mu, float sigma) {
     if (h->d > 0 && (!mu || !aligned16(mu))) return RELAY_EINVAL;
     h->mu = mu;
     h->sigma = sigma;
+    h->obj.source = relaysum::kMuStored;
+    h->has_objective = true;
+    return RELAY_OK;
+}
+
+int relay_set_objective_generated(relay_handle* h, const float* mix, int32_t K, float mu_scale,
+                                  uint64_t mu_seed, float sigma) {
+    if (!h || K < 0 || (K > 0 && !mix) || !std::isfinite(mu_scale) || !std::isfinite(sigma) ||
+        sigma < 0.0f)
+        return RELAY_EINVAL;
+    if (K > 32767) return RELAY_EUNSUPPORTED;
+    const int n = h->prog.n;
+    Objective o;
+    std::memset(&o, 0, sizeof(o));
+    int nnz = 0;
+    for (int i = 0; i < n; ++i) {
+        o.row_off[i] = static_cast<int16_t>(nnz);
+        for (int k = 0; k < K; ++k) {
+            const float w = mix[static_cast<int64_t>(i) * K + k];
+            if (!std::isfinite(w)) return RELAY_EINVAL;
+            if (w == 0.0f) continue;
+            if (nnz >= relaysum::kMaxMixNnz) return RELAY_EUNSUPPORTED;
+            o.col[nnz] = static_cast<int16_t>(k);
+            o.w[nnz] = w;
+            ++nnz;
+        }
+    }
+    o.row_off[n] = static_cast<int16_t>(nnz);
+    o.K = K;
+    o.scale = mu_scale;
+    o.k0 = static_cast<uint32_t>(mu_seed);
+    o.k1 = static_cast<uint32_t>(mu_seed >> 32);
+    // one Philox block per non-zero, or K per quad when that is fewer
+    o.source = (K <= relaysum::kMaxCachedCentres && K < nnz) ? relaysum::kMuCachedCentres
+                                                              : relaysum::kMuPerRow;
+    h->obj = o;
+    h->mu = nullptr;
+    h->sigma = sigma;
     h->has_objective = true;
     return RELAY_OK;
 }
@@ -484,9 +620,9 @@ int relay_fill_objective(relay_handle* h, float* mu, const float* mix, int32_t K
     if (h->d == 0) return RELAY_OK;
     if (!mu || !aligned16(mu) || (K > 0 && !mix)) return RELAY_EINVAL;
     const int threads = 256;
-    relay_fill_mu_kernel<<<grid_for(h->ld / 4, threads), threads, 0, stream>>>(
-        mu, mix, h->prog.n, K, h->ld, h->d, static_cast<uint32_t>(h->c0 / 4), mu_scale,
-        static_cast<uint32_t>(mu_seed), static_cast<uint32_t>(mu_seed >> 32));
+    relay_fill_mu_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
+        mu, mix, h->prog.n, K, h->ld_x, h->nquads, h->d, static_cast<uint32_t>(h->c0 / 4), mu_scale,
+        philox_key(mu_seed));
     return launch_status();
 }
 
@@ -501,10 +637,9 @@ int relay_init(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* c
     if (E > 0 && cudaMemsetAsync(counts, 0, sizeof(int32_t) * E, stream) != cudaSuccess) return RELAY_ECUDA;
     if (h->d == 0) return RELAY_OK;
     const int threads = 256;
-    relay_init_kernel<<<grid_for(h->ld / 4, threads), threads, 0, stream>>>(
-        x, E > 0 ? msg_a : nullptr, E > 0 ? msg_b : nullptr, h->prog.n, E, h->ld, h->d,
-        static_cast<uint32_t>(h->c0 / 4), x0_std, static_cast<uint32_t>(seed),
-        static_cast<uint32_t>(seed >> 32));
+    relay_init_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
+        x, E > 0 ? msg_a : nullptr, E > 0 ? msg_b : nullptr, h->prog.n, E, h->ld_x, h->ld_m, h->nquads,
+        h->d, static_cast<uint32_t>(h->c0 / 4), x0_std, philox_key(seed));
     return launch_status();
 }
 
@@ -528,15 +663,15 @@ int relay_step_models(relay_handle* h, float* x, const float* msg_in, float* msg
     a.msg_in = msg_in;
     a.msg_out = msg_out;
     a.counts = counts;
-    a.ld = h->ld;
+    a.ld_x = h->ld_x;
+    a.ld_m = h->ld_m;
     a.nquads = h->nquads;
     a.q0 = static_cast<uint32_t>(h->c0 / 4);
     a.step = static_cast<uint32_t>(step);
-    a.k0 = static_cast<uint32_t>(seed);
-    a.k1 = static_cast<uint32_t>(seed >> 32);
+    a.key = philox_key(seed);
     a.lr = lr;
     a.sigma = h->sigma;
-    return h->mode == 0 ? launch_models<0>(h, a, stream) : launch_models<1>(h, a, stream);
+    return h->mode == 0 ? launch_models_obj<0>(h, a, stream) : launch_models_obj<1>(h, a, stream);
 }
 
 int relay_step(relay_handle* h, float* x, const float* msg_in, float* msg_out, int32_t* counts, float lr,
@@ -570,9 +705,9 @@ int relay_program(const relay_handle* h, int32_t* nslots, int32_t* order, int32_
         if (order) order[i] = p.order[i];
         if (node_rec) {
             const NodeRec& r = p.node[i];
-            const int32_t v[8] = {r.deg, r.pos_base, r.parent_pos, r.recv_slot,
-                                  r.acc_slot, r.parent_acc, r.fin_parent, r.parent};
-            std::memcpy(node_rec + 8 * i, v, sizeof(v));
+            const int32_t v[10] = {r.deg,        r.pos_base,   r.parent_pos, r.recv_slot, r.acc_slot,
+                                   r.parent_acc, r.fin_parent, r.parent,     r.tot_slot,  r.flags};
+            std::memcpy(node_rec + 10 * i, v, sizeof(v));
         }
     }
     if (pos_rec)

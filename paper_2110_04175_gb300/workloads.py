@@ -32,6 +32,43 @@ def binary_tree(n: int) -> np.ndarray:
     return np.array([((i - 1) // 2, i) for i in range(1, n)], dtype=np.int32).reshape(-1, 2)
 
 
+def inorder_binary_tree(n: int) -> np.ndarray:
+    """Binary tree on 0..n-1 in in-order labelling: rank r has label v = r + 1
+    in the complete binary tree whose node v sits at height ctz(v); its parent
+    is the nearest ancestor with a label <= n.  Every even rank is a leaf and
+    every odd rank has a child, so each node has at most three edges."""
+    if n <= 1:
+        return np.zeros((0, 2), dtype=np.int32)
+    top = 1 << (n.bit_length() - 1)          # root label: largest power of two <= n
+    edges = []
+    for v in range(1, n + 1):
+        if v == top:
+            continue
+        p = v
+        while True:
+            h = (p & -p).bit_length() - 1    # height of p
+            up, down = p + (1 << h), p - (1 << h)
+            p = up if (up >> (h + 1)) & 1 else down   # the neighbour label with ctz = h + 1
+            if p <= n:
+                break
+        edges.append((min(v, p) - 1, max(v, p) - 1))
+    return np.array(sorted(edges), dtype=np.int32)
+
+
+def double_binary_trees(n: int):
+    """The two complementary trees of Section 3 ("Spanning trees"): tree A is
+    the in-order binary tree, tree B its mirror image r -> n-1-r (n even) or
+    its shift r -> r+1 mod n (n odd), so that the internal nodes of one tree
+    are leaves of the other."""
+    a = inorder_binary_tree(n)
+    if n % 2 == 0:
+        b = (n - 1) - a
+    else:
+        b = (a + 1) % n
+    b = np.sort(b, axis=1)
+    return a, np.array(sorted(map(tuple, b)), dtype=np.int32).reshape(-1, 2)
+
+
 def star(n: int, hub: int = 0) -> np.ndarray:
     """Star: the hub is connected to every other worker."""
     return np.array([(hub, i) for i in range(n) if i != hub], dtype=np.int32).reshape(-1, 2)
@@ -116,7 +153,8 @@ def dirichlet_mix(n: int, K: int, alpha: float, seed: int = 0) -> np.ndarray:
 class Workload:
     name: str
     n: int
-    edges: np.ndarray      # (n-1, 2) int32 undirected tree edges
+    edges: np.ndarray      # (n-1, 2) int32 undirected tree edges, or a list of
+                           # trees splitting the coordinates (double binary trees)
     d: int                 # parameters per worker
     mix: np.ndarray        # (n, K) float32 mixture of Gaussian centres
     mu_scale: float        # mu_i = mu_scale * sum_k mix[i, k] N_k
@@ -173,9 +211,17 @@ def sweep64(shape: str) -> Workload:
                     0.05, 0.05, 0.0, 100)
 
 
+def double16_vgg11() -> Workload:
+    """16 workers on double binary trees (Section 3), VGG-11-sized vector: the
+    paper's data-centre topology for its 16-worker experiments."""
+    n = 16
+    return Workload("double16_d9231114", n, list(double_binary_trees(n)), 9_231_114,
+                    identity_mix(n), 1.0, 0.05, 0.05, 0.0, 200)
+
+
 def all_workloads() -> list:
     return [chain8_d4096(), binary16_resnet20(), chain16_vgg11(), binary32_bert()] + [
-        sweep64(s) for s in ("star", "chain", "binary", "torus")]
+        sweep64(s) for s in ("star", "chain", "binary", "torus")] + [double16_vgg11()]
 
 
 def by_name(name: str) -> Workload:
