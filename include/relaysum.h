@@ -93,6 +93,26 @@ int relay_edges(const relay_handle *h, int32_t *src, int32_t *dst);
  * passed to later calls must stay 16-byte aligned.  Default: relay_ld(h). */
 int relay_set_strides(relay_handle *h, int64_t ld_x, int64_t ld_msg);
 
+#define RELAY_OPT_SGD 0       /* x^{t+1/2} = x^t - lr g                                  */
+#define RELAY_OPT_NESTEROV 1  /* m = beta1 m + g; x^{t+1/2} = x^t - lr (g + beta1 m)     */
+#define RELAY_OPT_ADAM 2      /* PyTorch's Adam (no weight decay), bias-corrected at t+1 */
+
+/* Local optimiser of Alg. 1's local step (appendix "RelaySGD with
+ * momentum", "RelaySGD with Adam"; all state is local to each worker).
+ * state1 (Nesterov: m; Adam: first moment) and state2 (Adam: second moment)
+ * are caller-owned device fp32 [n][ld_x] arrays with the stride of x,
+ * read and written by every step; relay_init zeroes them.  Nesterov needs
+ * 0 <= beta1 < 1; Adam 0 <= beta1, beta2 < 1 and eps > 0.  Default SGD. */
+int relay_set_local_optimizer(relay_handle *h, int32_t kind, float beta1, float beta2, float eps,
+                              float *state1, float *state2);
+
+/* Messages lost in transit (Section 4.4, "Robustness to unreliable
+ * communication"): host uint8 [E], non-zero = the message sent on that
+ * directed edge by every later step never arrives, so its receiver reads
+ * m = 0 and c = 0 (and relays those).  NULL clears.  The mask is copied into
+ * the launch arguments of each step: change it between steps freely. */
+int relay_set_lost_messages(relay_handle *h, const uint8_t *lost);
+
 /* Rebuild rule: 0 = Algorithm 1 (divide by nbar), 1 = robust rule of
  * Section 4.4 (fill the n - nbar missing models with x_i^t, divide by n).
  * The default is 1. */

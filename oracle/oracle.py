@@ -72,10 +72,24 @@ def _load():
                                    ctypes.c_double, ctypes.c_uint64, ctypes.c_int64,
                                    ctypes.c_int64, ctypes.c_int, i32p]
         lib.oracle_run.restype = ctypes.c_int
+        lib.oracle_run_ext.argtypes = [ctypes.c_int, i32p, ctypes.c_int, ctypes.c_int64,
+                                       ctypes.c_int64, f64p, f64p, f64p, i32p, f64p, f64p,
+                                       ctypes.c_double, ctypes.c_double, ctypes.c_uint64,
+                                       ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
+                                       ctypes.POINTER(_Opts), i32p]
+        lib.oracle_run_ext.restype = ctypes.c_int
         lib.oracle_edges.argtypes = [ctypes.c_int, i32p, ctypes.c_int, i32p, i32p]
         lib.oracle_edges.restype = ctypes.c_int
         _lib = lib
         return lib
+
+
+class _Opts(ctypes.Structure):
+    _fields_ = [("opt", ctypes.c_int), ("beta1", ctypes.c_double), ("beta2", ctypes.c_double),
+                ("eps", ctypes.c_double), ("drop", ctypes.POINTER(ctypes.c_uint8))]
+
+
+OPT_SGD, OPT_NESTEROV, OPT_ADAM = 0, 1, 2
 
 
 def _ptr(a: np.ndarray, ctype):
@@ -178,6 +192,41 @@ def run(n: int, edge_list, x: np.ndarray, mu: np.ndarray, msg: np.ndarray, count
     return nbar
 
 
+def run_ext(n: int, edge_list, x, mu, msg, counts, lr: float, sigma: float, seed: int,
+            step0: int, steps: int, mode: int = 0, c0: int = 0, opt: int = OPT_SGD,
+            beta1: float = 0.0, beta2: float = 0.0, eps: float = 0.0, s1=None, s2=None,
+            drop=None):
+    """run() with a local optimiser (SGD / Nesterov momentum / Adam, state
+    arrays s1, s2 [n][len] in place) and an optional mask drop[steps][E] of
+    lost messages."""
+    lib = _load()
+    e = _edges_arr(edge_list)
+    E = 2 * e.shape[0]
+    length = x.shape[1]
+    for a, rows in ((x, n), (mu, n), (msg, E)):
+        assert a.dtype == np.float64 and a.flags.c_contiguous and a.shape == (rows, length)
+    for a in (s1, s2):
+        if a is not None:
+            assert a.dtype == np.float64 and a.flags.c_contiguous and a.shape == (n, length)
+    assert counts.dtype == np.int32 and counts.shape == (E,)
+    o = _Opts(opt, beta1, beta2, eps, None)
+    if drop is not None:
+        drop = np.ascontiguousarray(np.asarray(drop, dtype=np.uint8).reshape(steps, E))
+        o.drop = drop.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8))
+    nbar = np.zeros(n, dtype=np.int32)
+    msg_p = msg if E > 0 else np.zeros((1, max(length, 1)))
+    cnt_p = counts if E > 0 else np.zeros(1, dtype=np.int32)
+    null = ctypes.POINTER(ctypes.c_double)()
+    _check(lib.oracle_run_ext(n, _ptr(e, ctypes.c_int32), e.shape[0], c0, length,
+                              _ptr(x, ctypes.c_double), _ptr(mu, ctypes.c_double),
+                              _ptr(msg_p, ctypes.c_double), _ptr(cnt_p, ctypes.c_int32),
+                              _ptr(s1, ctypes.c_double) if s1 is not None else null,
+                              _ptr(s2, ctypes.c_double) if s2 is not None else null,
+                              float(lr), float(sigma), seed, step0, steps, mode, ctypes.byref(o),
+                              _ptr(nbar, ctypes.c_int32)))
+    return nbar
+
+
 class State:
     """Oracle-side state of a RelaySum run on coordinate slice [c0, c0+len)."""
 
@@ -200,9 +249,21 @@ class State:
         self.msg[:] = 0.0
         self.counts[:] = 0
         self.step = 0
+        self.s1 = np.zeros((self.n, self.length))
+        self.s2 = np.zeros((self.n, self.length))
 
-    def advance(self, steps: int, lr: float, sigma: float, seed: int, mode: int = 0):
-        nbar = run(self.n, self.edges, self.x, self.mu, self.msg, self.counts, lr, sigma, seed,
-                   self.step, steps, mode, self.c0)
+    def advance(self, steps: int, lr: float, sigma: float, seed: int, mode: int = 0,
+                opt: int = OPT_SGD, beta1: float = 0.0, beta2: float = 0.0, eps: float = 0.0,
+                drop=None):
+        if opt == OPT_SGD and drop is None:
+            nbar = run(self.n, self.edges, self.x, self.mu, self.msg, self.counts, lr, sigma,
+                       seed, self.step, steps, mode, self.c0)
+        else:
+            if not hasattr(self, "s1"):
+                self.s1 = np.zeros((self.n, self.length))
+                self.s2 = np.zeros((self.n, self.length))
+            nbar = run_ext(self.n, self.edges, self.x, self.mu, self.msg, self.counts, lr, sigma,
+                           seed, self.step, steps, mode, self.c0, opt, beta1, beta2, eps,
+                           self.s1, self.s2, drop)
         self.step += steps
         return nbar

@@ -232,24 +232,37 @@ int oracle_fill_x0(int n, double x0_std, uint64_t seed, int64_t c0, int64_t len,
 
 /* ------------------------------------------------------------ the steps */
 
-/* Runs `steps` iterations t = step0 .. step0+steps-1 of Algorithm 1 on the
- * coordinate slice [c0, c0+len) of every worker.
+/* Options beyond plain Algorithm 1.
  *
- *   x      [n][len]  in: x^{step0}            out: x^{step0+steps}
- *   mu     [n][len]  the quadratic centres mu_i
- *   msg    [E][len]  in: m^{step0-1}          out: m^{step0+steps-1}
- *   counts [E]       in: c^{step0-1}          out: c^{step0+steps-1}
- *   nbar   [n]       out: nbar^{step0+steps} (may be NULL)
+ * Local optimiser (replaces the local-step line of Alg. 1):
+ *   opt 0  SGD:       x^{t+1/2} = x^t - lr g^t
+ *   opt 1  Nesterov momentum (appendix "RelaySGD with momentum"), s1 = m,
+ *          m^{-1} = 0:  m^t = beta1 m^{t-1} + g^t,
+ *                       x^{t+1/2} = x^t - lr (g^t + beta1 m^t)
+ *   opt 2  Adam (appendix "RelaySGD with Adam": PyTorch's standard Adam, all
+ *          state local), s1 = m, s2 = v, both 0 at t = 0, k = t + 1:
+ *          m = beta1 m + (1 - beta1) g,  v = beta2 v + (1 - beta2) g^2,
+ *          x^{t+1/2} = x^t - (lr / (1 - beta1^k)) m / (sqrt(v) / sqrt(1 - beta2^k) + eps)
+ * where g^t = (x^t - mu) + sigma xi^t.
  *
- * Coordinates never interact (every line of Alg. 1 is per coordinate) and
- * the noise is keyed by the absolute coordinate, so any slice reproduces
- * exactly the values of the full vector.  len == 0 runs the counters only. */
-int oracle_run(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t len,
-               double *x, const double *mu, double *msg, int32_t *counts,
-               double lr, double sigma, uint64_t seed, int64_t step0,
-               int64_t steps, int mode, int32_t *nbar) {
-    if (len < 0 || c0 < 0 || step0 < 0 || steps < 0 || (mode != 0 && mode != 1))
+ * Lost messages (Section 4.4, Table 5): drop[(t - step0) * E + e] != 0 means
+ * the message sent on directed edge e at step t never arrives: its receiver
+ * sees m = 0 and c = 0, uses them in its rebuild and relays them onwards. */
+typedef struct {
+    int opt;
+    double beta1, beta2, eps;
+    const uint8_t *drop;  /* [steps][E] or NULL */
+} oracle_opts;
+
+int oracle_run_ext(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t len,
+                   double *x, const double *mu, double *msg, int32_t *counts, double *s1,
+                   double *s2, double lr, double sigma, uint64_t seed, int64_t step0,
+                   int64_t steps, int mode, const oracle_opts *opts, int32_t *nbar) {
+    const int opt = opts ? opts->opt : 0;
+    if (len < 0 || c0 < 0 || step0 < 0 || steps < 0 || (mode != 0 && mode != 1) || opt < 0 ||
+        opt > 2)
         return ORACLE_EINVAL;
+    if ((opt >= 1 && !s1) || (opt == 2 && !s2)) return ORACLE_EINVAL;
     if (step0 + steps > 4294967296LL) return ORACLE_EINVAL;
     otree t;
     int rc = otree_build(n, edges, n_edges, &t);
@@ -264,13 +277,14 @@ int oracle_run(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t len
         return ORACLE_ENOMEM;
     }
     for (int64_t t_step = step0; t_step < step0 + steps; ++t_step) {
+        const uint8_t *lost = (opts && opts->drop) ? opts->drop + (t_step - step0) * E : NULL;
         /* counters c^{t} from c^{t-1} */
         for (int e = 0; e < E; ++e) {
             int i = t.src[e], j = t.dst[e];
             int32_t s = 1;
             for (int k = t.nbr_off[i]; k < t.nbr_off[i + 1]; ++k)
                 if (t.nbr[k] != j) s += counts[t.in_edge[k]];
-            c_new[e] = s;
+            c_new[e] = (lost && lost[e]) ? 0 : s;
         }
         memcpy(counts, c_new, sizeof(int32_t) * (size_t)E);
         /* nbar^{t+1} from c^{t} */
@@ -280,12 +294,26 @@ int oracle_run(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t len
             nb[i] = s;
         }
         /* local step */
+        const double k_adam = (double)(t_step + 1);
         for (int i = 0; i < n; ++i)
             for (int64_t c = 0; c < len; ++c) {
-                double xv = x[(int64_t)i * len + c];
+                const int64_t ic = (int64_t)i * len + c;
+                double xv = x[ic];
                 double xi = oracle_normal(seed, c0 + c, (uint32_t)i, (uint32_t)t_step, 0u);
-                double g = (xv - mu[(int64_t)i * len + c]) + sigma * xi;
-                xh[(int64_t)i * len + c] = xv - lr * g;
+                double g = (xv - mu[ic]) + sigma * xi;
+                if (opt == 0) {
+                    xh[ic] = xv - lr * g;
+                } else if (opt == 1) {
+                    s1[ic] = opts->beta1 * s1[ic] + g;
+                    xh[ic] = xv - lr * (g + opts->beta1 * s1[ic]);
+                } else {
+                    const double b1 = opts->beta1, b2 = opts->beta2;
+                    s1[ic] = b1 * s1[ic] + (1.0 - b1) * g;
+                    s2[ic] = b2 * s2[ic] + (1.0 - b2) * g * g;
+                    const double bc1 = 1.0 - pow(b1, k_adam), bc2 = 1.0 - pow(b2, k_adam);
+                    const double denom = sqrt(s2[ic]) / sqrt(bc2) + opts->eps;
+                    xh[ic] = xv - (lr / bc1) * s1[ic] / denom;
+                }
             }
         /* relay messages m^{t} from x^{t+1/2} and m^{t-1} */
         for (int e = 0; e < E; ++e) {
@@ -294,7 +322,7 @@ int oracle_run(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t len
                 double s = xh[(int64_t)i * len + c];
                 for (int k = t.nbr_off[i]; k < t.nbr_off[i + 1]; ++k)
                     if (t.nbr[k] != j) s += msg[(int64_t)t.in_edge[k] * len + c];
-                m_new[(int64_t)e * len + c] = s;
+                m_new[(int64_t)e * len + c] = (lost && lost[e]) ? 0.0 : s;
             }
         }
         /* rebuild x^{t+1} */
@@ -322,6 +350,26 @@ int oracle_run(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t len
     }
     free(c_new); free(nb); free(xh); free(m_new); otree_free(&t);
     return ORACLE_OK;
+}
+
+/* Runs `steps` iterations t = step0 .. step0+steps-1 of Algorithm 1 on the
+ * coordinate slice [c0, c0+len) of every worker.
+ *
+ *   x      [n][len]  in: x^{step0}            out: x^{step0+steps}
+ *   mu     [n][len]  the quadratic centres mu_i
+ *   msg    [E][len]  in: m^{step0-1}          out: m^{step0+steps-1}
+ *   counts [E]       in: c^{step0-1}          out: c^{step0+steps-1}
+ *   nbar   [n]       out: nbar^{step0+steps} (may be NULL)
+ *
+ * Coordinates never interact (every line of Alg. 1 is per coordinate) and
+ * the noise is keyed by the absolute coordinate, so any slice reproduces
+ * exactly the values of the full vector.  len == 0 runs the counters only. */
+int oracle_run(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t len,
+               double *x, const double *mu, double *msg, int32_t *counts,
+               double lr, double sigma, uint64_t seed, int64_t step0,
+               int64_t steps, int mode, int32_t *nbar) {
+    return oracle_run_ext(n, edges, n_edges, c0, len, x, mu, msg, counts, NULL, NULL, lr, sigma,
+                          seed, step0, steps, mode, NULL, nbar);
 }
 
 /* Directed edge table of the oracle's own numbering, for cross-checks. */

@@ -16,6 +16,9 @@ RELAY_ECUDA = -3
 RELAY_ENOMEM = -4
 RELAY_EUNSUPPORTED = -5
 RELAY_MAX_N = 256
+RELAY_OPT_SGD = 0
+RELAY_OPT_NESTEROV = 1
+RELAY_OPT_ADAM = 2
 
 _lock = threading.Lock()
 _lib = None
@@ -45,6 +48,8 @@ def _load():
             "relay_edges": (ctypes.c_int, [vp, vp, vp]),
             "relay_set_rebuild_mode": (ctypes.c_int, [vp, i32]),
             "relay_set_strides": (ctypes.c_int, [vp, i64, i64]),
+            "relay_set_local_optimizer": (ctypes.c_int, [vp, i32, f32, f32, f32, vp, vp]),
+            "relay_set_lost_messages": (ctypes.c_int, [vp, vp]),
             "relay_set_coord_offset": (ctypes.c_int, [vp, i64]),
             "relay_set_objective": (ctypes.c_int, [vp, vp, f32]),
             "relay_set_objective_generated": (ctypes.c_int, [vp, vp, i32, f32, u64, f32]),
@@ -169,6 +174,23 @@ def relay_set_strides(h, ld_x: int, ld_msg: int):
     _check(_load().relay_set_strides(_h(h), int(ld_x), int(ld_msg)), "relay_set_strides")
 
 
+def relay_set_local_optimizer(h, kind: int, beta1: float = 0.0, beta2: float = 0.0,
+                              eps: float = 0.0, state1=None, state2=None):
+    _check(_load().relay_set_local_optimizer(_h(h), int(kind), float(beta1), float(beta2),
+                                             float(eps), _ptr(state1), _ptr(state2)),
+           "relay_set_local_optimizer")
+
+
+def relay_set_lost_messages(h, lost=None):
+    """lost: host array of E flags (non-zero = lost) or None."""
+    if lost is None:
+        _check(_load().relay_set_lost_messages(_h(h), None), "relay_set_lost_messages")
+        return
+    m = np.ascontiguousarray(np.asarray(lost, dtype=np.uint8))
+    _check(_load().relay_set_lost_messages(_h(h), m.ctypes.data if m.size else None),
+           "relay_set_lost_messages")
+
+
 def relay_set_coord_offset(h, c0: int):
     _check(_load().relay_set_coord_offset(_h(h), int(c0)), "relay_set_coord_offset")
 
@@ -264,7 +286,8 @@ class RelayRun:
     """
 
     def __init__(self, n: int, d: int, edges, device="cuda", mode: int = 1, c0: int = 0,
-                 objective: str = "stored"):
+                 objective: str = "stored", optimizer=None):
+        """optimizer: None (SGD), ("nesterov", beta1) or ("adam", beta1, beta2, eps)."""
         import torch
         if objective not in ("stored", "generated"):
             raise ValueError(objective)
@@ -276,6 +299,9 @@ class RelayRun:
         f32 = dict(dtype=torch.float32, device=self.device)
         self.x = torch.empty(n, self.ld, **f32)
         self.mu = torch.empty(n, self.ld, **f32) if objective == "stored" else None
+        kind = {None: RELAY_OPT_SGD, "nesterov": RELAY_OPT_NESTEROV, "adam": RELAY_OPT_ADAM}[
+            optimizer[0] if optimizer else None]
+        self.state = [torch.empty(n, self.ld, **f32) for _ in range(kind)]  # m (and v)
         nq = (d + 3) // 4
         self.trees = []
         for k, tree_edges in enumerate(trees):
@@ -287,6 +313,10 @@ class RelayRun:
             relay_set_coord_offset(h, c0 + col0)
             ld_m = relay_ld(h)
             relay_set_strides(h, self.ld, ld_m)
+            if kind != RELAY_OPT_SGD:
+                hyper = list(optimizer[1:]) + [0.0] * (3 - len(optimizer[1:]))
+                st = [_window_ptr(t, col0) if dk > 0 else None for t in self.state] + [None]
+                relay_set_local_optimizer(h, kind, hyper[0], hyper[1], hyper[2], st[0], st[1])
             E = relay_num_edges(h)
             msg = [torch.empty(max(E, 1), max(ld_m, 1), **f32) for _ in range(2)]
             counts = torch.zeros(max(E, 1), dtype=torch.int32, device=self.device)
@@ -343,6 +373,10 @@ class RelayRun:
             tr.cur = 0
         self._mix = mix_t  # keep alive until the fills have run
         self.t = 0
+
+    def set_lost(self, lost, tree: int = 0):
+        """Messages of the next steps lost in transit on tree `tree` (E flags or None)."""
+        relay_set_lost_messages(self.trees[tree].h, lost)
 
     def step(self, lr: float, seed: int, stream=None):
         for tr in self.trees:

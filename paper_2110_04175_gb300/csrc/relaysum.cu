@@ -44,6 +44,14 @@ struct relay_handle {
     const float* mu = nullptr;
     float sigma = 0.0f;
     bool has_objective = false;
+    // local optimiser of Alg. 1's local step (appendix "RelaySGD with momentum / Adam")
+    int32_t opt = 0;
+    float beta1 = 0.0f, beta2 = 0.0f, eps = 0.0f;
+    float* s1 = nullptr;  // momentum buffer / Adam first moment, [n][ld_x]
+    float* s2 = nullptr;  // Adam second moment, [n][ld_x]
+    // messages lost in transit (Section 4.4), one bit per directed edge
+    bool has_lost = false;
+    uint32_t lost[relaysum::kMaxE / 32 + 1] = {};
 };
 
 namespace {
@@ -132,9 +140,13 @@ __device__ __forceinline__ float4 scale4_rn(float4 a, float s) {
 __device__ __forceinline__ float4 fma4(float w, float4 z, float4 acc) {
     return make_float4(fmaf(w, z.x, acc.x), fmaf(w, z.y, acc.y), fmaf(w, z.z, acc.z), fmaf(w, z.w, acc.w));
 }
-// Loads read once per step stream through L2 with evict-first priority.
+// Loads read once per step: read-only path, no L1 allocation.
 __device__ __forceinline__ float4 ld_stream(const float* p) {
-    return __ldcs(reinterpret_cast<const float4*>(p));
+    float4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "l"(p));
+    return v;
 }
 // A wide node's incoming messages are read again at its children's visits
 // (program.h): keep them in L2 with evict-last priority until then.
@@ -155,8 +167,14 @@ __device__ __forceinline__ void st_stream(float* p, float4 v) {
 // ------------------------------------------------------------------ counters
 
 // c^t_{i->j} = 1 + sum_{k in N(i)\j} c^{t-1}_{k->i}: the incoming edge from
-// j is e ^ 1 for e = i -> j.
-__global__ void relay_counts_kernel(const __grid_constant__ Program prog, int32_t* counts) {
+// j is e ^ 1 for e = i -> j.  A lost message (Section 4.4) arrives as c = 0.
+struct LostMask {
+    uint32_t w[relaysum::kMaxE / 32 + 1];
+    __host__ __device__ __forceinline__ bool operator()(int e) const { return (w[e >> 5] >> (e & 31)) & 1u; }
+};
+
+__global__ void relay_counts_kernel(const __grid_constant__ Program prog, const __grid_constant__ LostMask lost,
+                                    int has_lost, int32_t* counts) {
     __shared__ int32_t c_old[kMaxE];
     const int E = prog.E;
     for (int e = threadIdx.x; e < E; e += blockDim.x) c_old[e] = counts[e];
@@ -168,7 +186,7 @@ __global__ void relay_counts_kernel(const __grid_constant__ Program prog, int32_
             const int in = prog.pos_in[r.pos_base + p];
             if (in != (e ^ 1)) s += c_old[in];
         }
-        counts[e] = s;
+        counts[e] = (has_lost && lost(e)) ? 0 : s;  // a lost message carries no count
     }
 }
 
@@ -186,8 +204,21 @@ struct ModelArgs {
     uint32_t q0;      // absolute quad of local coordinate 0
     uint32_t step;
     float lr, sigma;
+    int mode;         // 0: Alg. 1 rebuild, 1: robust rebuild
+    int has_lost;     // any bit of `lost` set
+    LostMask lost;    // messages lost in transit this step
+    float* s1;        // optimiser state (momentum / Adam m), [n][ld_x]
+    float* s2;        // Adam v, [n][ld_x]
+    float beta1, beta2, eps;
+    float adam_step;  // lr / (1 - beta1^{t+1})
+    float adam_ibc2;  // 1 / sqrt(1 - beta2^{t+1})
     PhiloxKey key;    // noise key schedule
 };
+
+// A lost message reaches its receiver as zero (Section 4.4).
+__device__ __forceinline__ float4 delivered(const ModelArgs& a, int e, float4 m) {
+    return (a.has_lost && a.lost(e)) ? make_float4(0.f, 0.f, 0.f, 0.f) : m;
+}
 
 // Per-thread view of the shared-memory slots: slot s of this thread is
 // base[s * stride]; a warp's 32 float4 of one slot are contiguous.
@@ -228,8 +259,9 @@ __device__ __forceinline__ void visit_small(const Program& prog, const NodeRec& 
     for (int s = D - 2; s >= 0; --s) suf[s] = add4(m[s], suf[s + 1]);
 #pragma unroll
     for (int s = 0; s < D; ++s) {
-        const float4 out = (s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]);
-        st_stream(a.msg_out + prog.pos_out[r.pos_base + s] * a.ld_m + 4 * q, out);
+        const int e = prog.pos_out[r.pos_base + s];
+        const float4 out = delivered(a, e, (s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]));
+        st_stream(a.msg_out + e * a.ld_m + 4 * q, out);
         if (s == r.parent_pos) {
             to_parent(r, a, q, out, sl, s_scale);
         } else {
@@ -254,11 +286,47 @@ __device__ __noinline__ void visit_wide(const Program& prog, const NodeRec& r, c
         if (s == r.parent_pos) from_parent = m;
     }
     if (r.parent_pos >= 0) {
-        const float4 out = sub4(total, from_parent);
-        st_stream(a.msg_out + prog.pos_out[base + r.parent_pos] * a.ld_m + 4 * q, out);
+        const int e = prog.pos_out[base + r.parent_pos];
+        const float4 out = delivered(a, e, sub4(total, from_parent));
+        st_stream(a.msg_out + e * a.ld_m + 4 * q, out);
         to_parent(r, a, q, out, sl, s_scale);
     }
     sl[r.tot_slot] = total;
+}
+
+// Alg. 1's local step with the chosen optimiser, per coordinate.
+//   SGD:      x - lr g
+//   Nesterov: m = beta1 m + g;  x - lr (g + beta1 m)          (state s1 = m)
+//   Adam:     m = beta1 m + (1 - beta1) g;  v = beta2 v + (1 - beta2) g^2;
+//             x - adam_step m / (sqrt(v) adam_ibc2 + eps)     (s1 = m, s2 = v)
+__device__ __forceinline__ float sgd1(float lr, float x, float g) { return fmaf(-lr, g, x); }
+
+template <int OPT>
+__device__ __forceinline__ float4 local_step(const ModelArgs& a, int i, int64_t q, float4 x, float4 g) {
+    if (OPT == 0) return make_float4(sgd1(a.lr, x.x, g.x), sgd1(a.lr, x.y, g.y), sgd1(a.lr, x.z, g.z),
+                                     sgd1(a.lr, x.w, g.w));
+    float4* pm = reinterpret_cast<float4*>(a.s1 + i * a.ld_x + 4 * q);
+    float4 m = *pm;
+    if (OPT == 1) {
+        m = make_float4(fmaf(a.beta1, m.x, g.x), fmaf(a.beta1, m.y, g.y), fmaf(a.beta1, m.z, g.z),
+                        fmaf(a.beta1, m.w, g.w));
+        __stcs(pm, m);
+        return make_float4(fmaf(-a.lr, fmaf(a.beta1, m.x, g.x), x.x), fmaf(-a.lr, fmaf(a.beta1, m.y, g.y), x.y),
+                           fmaf(-a.lr, fmaf(a.beta1, m.z, g.z), x.z), fmaf(-a.lr, fmaf(a.beta1, m.w, g.w), x.w));
+    }
+    float4* pv = reinterpret_cast<float4*>(a.s2 + i * a.ld_x + 4 * q);
+    float4 v = *pv;
+    const float c1 = 1.0f - a.beta1, c2 = 1.0f - a.beta2;
+    m = make_float4(fmaf(a.beta1, m.x, c1 * g.x), fmaf(a.beta1, m.y, c1 * g.y), fmaf(a.beta1, m.z, c1 * g.z),
+                    fmaf(a.beta1, m.w, c1 * g.w));
+    v = make_float4(fmaf(a.beta2, v.x, c2 * g.x * g.x), fmaf(a.beta2, v.y, c2 * g.y * g.y),
+                    fmaf(a.beta2, v.z, c2 * g.z * g.z), fmaf(a.beta2, v.w, c2 * g.w * g.w));
+    __stcs(pm, m);
+    __stcs(pv, v);
+    auto upd = [&](float xx, float mm, float vv) {
+        return xx - a.adam_step * mm / fmaf(sqrtf(vv), a.adam_ibc2, a.eps);
+    };
+    return make_float4(upd(x.x, m.x, v.x), upd(x.y, m.y, v.y), upd(x.z, m.z, v.z), upd(x.w, m.w, v.w));
 }
 
 // mu_i for quad q: read, or regenerated exactly as relay_fill_mu_kernel
@@ -278,10 +346,11 @@ __device__ __forceinline__ float4 centre(const Objective& obj, const PhiloxKey& 
     return scale4_rn(acc, obj.scale);
 }
 
-// MODE 0: x' = acc / nbar (Alg. 1).  MODE 1: x' = (acc + (n - nbar) x) / n
+// mode 0: x' = acc / nbar (Alg. 1).  mode 1: x' = (acc + (n - nbar) x) / n
 // (robust rule), with the fill term folded into the accumulator up front.
-// OBJ: where mu comes from (ObjectiveSource).
-template <int MODE, int OBJ>
+// OBJ: where mu comes from (ObjectiveSource).  OPT: the local optimiser
+// (0 SGD, 1 Nesterov momentum, 2 Adam).
+template <int OBJ, int OPT>
 __global__ void __launch_bounds__(128)
 relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant__ Objective obj,
                     const __grid_constant__ PhiloxKey mu_key, const __grid_constant__ ModelArgs a) {
@@ -293,7 +362,7 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
         const NodeRec r = prog.node[i];
         int nbar = 1;
         for (int p = 0; p < r.deg; ++p) nbar += __ldg(a.counts + prog.pos_in[r.pos_base + p]);
-        if (MODE == 0) {
+        if (a.mode == 0) {
             s_scale[i] = 1.0f / static_cast<float>(nbar);
             s_fill[i] = 0.0f;
         } else {
@@ -319,21 +388,21 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
             const float4 mv = centre<OBJ>(obj, mu_key, a, i, q, cen, static_cast<int>(blockDim.x));
             const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i),
                                      a.step, 0u, a.key);
-            // x^{t+1/2} = x - lr * ((x - mu) + sigma * xi)
-            float4 xh;
-            xh.x = fmaf(-a.lr, fmaf(a.sigma, z.x, xv.x - mv.x), xv.x);
-            xh.y = fmaf(-a.lr, fmaf(a.sigma, z.y, xv.y - mv.y), xv.y);
-            xh.z = fmaf(-a.lr, fmaf(a.sigma, z.z, xv.z - mv.z), xv.z);
-            xh.w = fmaf(-a.lr, fmaf(a.sigma, z.w, xv.w - mv.w), xv.w);
+            // g = (x - mu) + sigma * xi, then the local optimiser's x^{t+1/2}
+            const float4 g = make_float4(fmaf(a.sigma, z.x, xv.x - mv.x), fmaf(a.sigma, z.y, xv.y - mv.y),
+                                         fmaf(a.sigma, z.z, xv.z - mv.z), fmaf(a.sigma, z.w, xv.w - mv.w));
+            const float4 xh = local_step<OPT>(a, i, q, xv, g);
             float4 acc = xh;
-            if (MODE == 1) acc = add4(scale4(xv, s_fill[i]), xh);
+            if (a.mode == 1) acc = add4(scale4(xv, s_fill[i]), xh);
             if (r.recv_slot >= 0) {
                 float4 recv = sl[r.recv_slot];
                 if (r.flags & relaysum::kRecvFromTotal) {
                     // m^t_{p->i} = T_p - m^{t-1}_{i->p}, written out here
                     const int pos = r.pos_base + r.parent_pos;
-                    recv = sub4(recv, ld_stream(a.msg_in + prog.pos_out[pos] * a.ld_m + 4 * q));
-                    st_stream(a.msg_out + prog.pos_in[pos] * a.ld_m + 4 * q, recv);
+                    const int e = prog.pos_in[pos];
+                    recv = delivered(a, e, sub4(recv, __ldg(reinterpret_cast<const float4*>(
+                                                          a.msg_in + prog.pos_out[pos] * a.ld_m + 4 * q))));
+                    st_stream(a.msg_out + e * a.ld_m + 4 * q, recv);
                 }
                 acc = add4(acc, recv);
             }
@@ -434,7 +503,7 @@ int models_threads(int nslots) {
     return t;
 }
 
-template <int MODE, int OBJ>
+template <int OBJ, int OPT>
 int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
     int dev = 0;
     const int sms = device_sms(&dev);
@@ -443,15 +512,17 @@ int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream
     const int threads = models_threads(per_thread);
     const size_t smem = static_cast<size_t>(per_thread) * threads * 16;
     if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
+    // opt in to the full shared memory once per device (the 48 KB default
+    // covers dynamic AND static shared memory)
     static std::atomic<bool> smem_set[kMaxDevices];
-    if (smem > 48 * 1024 && dev < kMaxDevices && !smem_set[dev].load()) {
-        if (cudaFuncSetAttribute(relay_models_kernel<MODE, OBJ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((dev >= kMaxDevices || !smem_set[dev].load())) {
+        if (cudaFuncSetAttribute(relay_models_kernel<OBJ, OPT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kMaxSmem) != cudaSuccess)
             return RELAY_ECUDA;
-        smem_set[dev].store(true);
+        if (dev < kMaxDevices) smem_set[dev].store(true);
     }
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_models_kernel<MODE, OBJ>, threads, smem) !=
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_models_kernel<OBJ, OPT>, threads, smem) !=
             cudaSuccess ||
         per_sm <= 0)
         return RELAY_ECUDA;
@@ -459,16 +530,16 @@ int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream
     const int64_t cap = static_cast<int64_t>(sms) * per_sm;
     const int grid = static_cast<int>(want < cap ? want : cap);
     const PhiloxKey mu_key = philox_key(static_cast<uint64_t>(h->obj.k0) | (static_cast<uint64_t>(h->obj.k1) << 32));
-    relay_models_kernel<MODE, OBJ><<<grid, threads, smem, stream>>>(h->prog, h->obj, mu_key, a);
+    relay_models_kernel<OBJ, OPT><<<grid, threads, smem, stream>>>(h->prog, h->obj, mu_key, a);
     return launch_status();
 }
 
-template <int MODE>
+template <int OPT>
 int launch_models_obj(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
     switch (h->obj.source) {
-        case relaysum::kMuStored: return launch_models<MODE, relaysum::kMuStored>(h, a, stream);
-        case relaysum::kMuPerRow: return launch_models<MODE, relaysum::kMuPerRow>(h, a, stream);
-        default: return launch_models<MODE, relaysum::kMuCachedCentres>(h, a, stream);
+        case relaysum::kMuStored: return launch_models<relaysum::kMuStored, OPT>(h, a, stream);
+        case relaysum::kMuPerRow: return launch_models<relaysum::kMuPerRow, OPT>(h, a, stream);
+        default: return launch_models<relaysum::kMuCachedCentres, OPT>(h, a, stream);
     }
 }
 
@@ -488,6 +559,9 @@ int check_step_args(const relay_handle* h, const float* x, const float* msg_in, 
     const int64_t mb = E > 0 ? ((E - 1) * h->ld_m + 4 * h->nquads) * 4 : 0;
     if (overlap(x, xb, msg_in, mb) || overlap(x, xb, msg_out, mb) || overlap(msg_in, mb, msg_out, mb))
         return RELAY_EINVAL;
+    for (const float* st : {static_cast<const float*>(h->s1), static_cast<const float*>(h->s2)})
+        if (st && (overlap(st, xb, x, xb) || overlap(st, xb, msg_in, mb) || overlap(st, xb, msg_out, mb)))
+            return RELAY_EINVAL;
     return RELAY_OK;
 }
 
@@ -551,6 +625,39 @@ int relay_set_strides(relay_handle* h, int64_t ld_x, int64_t ld_msg) {
     if (!h || ld_x < 4 * h->nquads || ld_msg < 4 * h->nquads || (ld_x & 3) || (ld_msg & 3)) return RELAY_EINVAL;
     h->ld_x = ld_x;
     h->ld_m = ld_msg;
+    return RELAY_OK;
+}
+
+int relay_set_local_optimizer(relay_handle* h, int32_t kind, float beta1, float beta2, float eps,
+                              float* state1, float* state2) {
+    if (!h || kind < RELAY_OPT_SGD || kind > RELAY_OPT_ADAM) return RELAY_EINVAL;
+    if (!std::isfinite(beta1) || !std::isfinite(beta2) || !std::isfinite(eps)) return RELAY_EINVAL;
+    if (kind == RELAY_OPT_NESTEROV && (beta1 < 0.0f || beta1 >= 1.0f)) return RELAY_EINVAL;
+    if (kind == RELAY_OPT_ADAM &&
+        (beta1 < 0.0f || beta1 >= 1.0f || beta2 < 0.0f || beta2 >= 1.0f || !(eps > 0.0f)))
+        return RELAY_EINVAL;
+    if (h->d > 0 && kind >= RELAY_OPT_NESTEROV && (!state1 || !aligned16(state1))) return RELAY_EINVAL;
+    if (h->d > 0 && kind == RELAY_OPT_ADAM && (!state2 || !aligned16(state2) || state2 == state1))
+        return RELAY_EINVAL;
+    h->opt = kind;
+    h->beta1 = beta1;
+    h->beta2 = beta2;
+    h->eps = eps;
+    h->s1 = kind >= RELAY_OPT_NESTEROV ? state1 : nullptr;
+    h->s2 = kind == RELAY_OPT_ADAM ? state2 : nullptr;
+    return RELAY_OK;
+}
+
+int relay_set_lost_messages(relay_handle* h, const uint8_t* lost) {
+    if (!h) return RELAY_EINVAL;
+    std::memset(h->lost, 0, sizeof(h->lost));
+    h->has_lost = false;
+    if (!lost) return RELAY_OK;
+    for (int e = 0; e < h->prog.E; ++e)
+        if (lost[e]) {
+            h->lost[e >> 5] |= 1u << (e & 31);
+            h->has_lost = true;
+        }
     return RELAY_OK;
 }
 
@@ -636,6 +743,13 @@ int relay_init(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* c
         return RELAY_EINVAL;
     if (E > 0 && cudaMemsetAsync(counts, 0, sizeof(int32_t) * E, stream) != cudaSuccess) return RELAY_ECUDA;
     if (h->d == 0) return RELAY_OK;
+    // optimiser state starts at zero (momentum buffer, Adam moments)
+    const size_t state_bytes = static_cast<size_t>((h->prog.n - 1) * h->ld_x + 4 * h->nquads) * 4;
+    for (float* st : {h->s1, h->s2})
+        if (st && cudaMemset2DAsync(st, static_cast<size_t>(h->ld_x) * 4, 0, static_cast<size_t>(4 * h->nquads) * 4,
+                                    static_cast<size_t>(h->prog.n), stream) != cudaSuccess)
+            return RELAY_ECUDA;
+    (void)state_bytes;
     const int threads = 256;
     relay_init_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
         x, E > 0 ? msg_a : nullptr, E > 0 ? msg_b : nullptr, h->prog.n, E, h->ld_x, h->ld_m, h->nquads,
@@ -647,7 +761,9 @@ int relay_step_counts(relay_handle* h, int32_t* counts, relay_stream_t stream) {
     if (!h) return RELAY_EINVAL;
     if (h->prog.E == 0) return RELAY_OK;
     if (!counts) return RELAY_EINVAL;
-    relay_counts_kernel<<<1, 256, 0, stream>>>(h->prog, counts);
+    LostMask lost;
+    std::memcpy(lost.w, h->lost, sizeof(lost.w));
+    relay_counts_kernel<<<1, 256, 0, stream>>>(h->prog, lost, h->has_lost ? 1 : 0, counts);
     return launch_status();
 }
 
@@ -671,7 +787,26 @@ int relay_step_models(relay_handle* h, float* x, const float* msg_in, float* msg
     a.key = philox_key(seed);
     a.lr = lr;
     a.sigma = h->sigma;
-    return h->mode == 0 ? launch_models_obj<0>(h, a, stream) : launch_models_obj<1>(h, a, stream);
+    a.mode = h->mode;
+    a.has_lost = h->has_lost ? 1 : 0;
+    std::memcpy(a.lost.w, h->lost, sizeof(a.lost.w));
+    a.s1 = h->s1;
+    a.s2 = h->s2;
+    a.beta1 = h->beta1;
+    a.beta2 = h->beta2;
+    a.eps = h->eps;
+    a.adam_step = 0.0f;
+    a.adam_ibc2 = 0.0f;
+    if (h->opt == 2) {  // bias corrections of step k = t + 1, in double
+        const double k = static_cast<double>(step) + 1.0;
+        a.adam_step = static_cast<float>(lr / (1.0 - std::pow(static_cast<double>(h->beta1), k)));
+        a.adam_ibc2 = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(static_cast<double>(h->beta2), k)));
+    }
+    switch (h->opt) {
+        case 0: return launch_models_obj<0>(h, a, stream);
+        case 1: return launch_models_obj<1>(h, a, stream);
+        default: return launch_models_obj<2>(h, a, stream);
+    }
 }
 
 int relay_step(relay_handle* h, float* x, const float* msg_in, float* msg_out, int32_t* counts, float lr,

@@ -1,0 +1,130 @@
+"""GPU parity of the extensions against the oracle: local momentum / Adam
+(appendix "RelaySGD with momentum / with Adam") and messages lost in transit
+with the robust rebuild (Section 4.4, Table 5)."""
+import gc
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2110_04175_gb300 as rs
+from oracle import oracle
+from paper_2110_04175_gb300 import build as rs_build
+from paper_2110_04175_gb300 import workloads as wl
+from tests.gpu_util import RTOL, parity_error, sample_columns
+
+pytestmark = pytest.mark.gpu
+
+OPTS = {"nesterov": (oracle.OPT_NESTEROV, ("nesterov", 0.9)),
+        "adam": (oracle.OPT_ADAM, ("adam", 0.9, 0.999, 1e-8))}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    rs_build.build()
+    yield
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+def _run_both(w, steps, mode, optimizer=None, lost=None, ranges=None, objective="stored"):
+    """GPU run through the C ABI and oracle runs on `ranges` (default: all
+    coordinates); lost: [steps][E] flags or None.  Returns the parity errors."""
+    run = rs.RelayRun(w.n, w.d, w.edges, device="cuda:0", mode=mode, objective=objective,
+                      optimizer=OPTS[optimizer][1] if optimizer else None)
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    for t in range(steps):
+        if lost is not None:
+            run.set_lost(lost[t])
+        run.step(w.lr, w.seed)
+    torch.cuda.synchronize()
+    ranges = ranges or [(0, w.d)]
+    kw = {}
+    if optimizer:
+        o = OPTS[optimizer]
+        kw = dict(opt=o[0], beta1=o[1][1], beta2=o[1][2] if len(o[1]) > 2 else 0.0,
+                  eps=o[1][3] if len(o[1]) > 3 else 0.0)
+    gx, gm, ox, om = [], [], [], []
+    counts = None
+    for start, length in ranges:
+        st = oracle.State(w.n, w.edges, length, c0=start)
+        st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+        lr, sigma = float(np.float32(w.lr)), float(np.float32(w.sigma))
+        if lost is None:
+            st.advance(steps, lr, sigma, w.seed, mode, **kw)
+        else:
+            for t in range(steps):
+                st.advance(1, lr, sigma, w.seed, mode, drop=lost[t:t + 1], **kw)
+        gx.append(run.x[:, start:start + length].double().cpu().numpy())
+        gm.append(run.messages[:run.E, start:start + length].double().cpu().numpy())
+        ox.append(st.x)
+        om.append(st.msg)
+        counts = st.counts
+    assert np.array_equal(run.counts[:run.E].cpu().numpy(), counts)
+    ex = parity_error(np.concatenate(gx, 1), np.concatenate(ox, 1))
+    em = parity_error(np.concatenate(gm, 1), np.concatenate(om, 1))
+    del run
+    gc.collect()
+    torch.cuda.empty_cache()
+    return ex, em
+
+
+@pytest.mark.parametrize("objective", ["stored", "generated"])
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("optimizer", ["nesterov", "adam"])
+@pytest.mark.parametrize("shape,n,d", [("chain", 8, 4096), ("star", 9, 1031), ("binary", 15, 2053),
+                                       ("single", 1, 517)])
+def test_local_optimizers_every_coordinate(shape, n, d, optimizer, mode, objective):
+    edges = {"chain": wl.chain(n), "star": wl.star(n), "binary": wl.binary_tree(n),
+             "single": np.zeros((0, 2), np.int32)}[shape]
+    w = wl.Workload(shape, n, edges, d, wl.identity_mix(n), 2.0, 0.1, 0.05, 0.1, 40)
+    ex, em = _run_both(w, w.steps, mode, optimizer, objective=objective)
+    assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+@pytest.mark.parametrize("optimizer", ["nesterov", "adam"])
+def test_local_optimizers_full_size_sampled(optimizer):
+    """The 32-worker 1.1e8-parameter workload with each local optimiser (50
+    steps), oracle on the first/last coordinates and 32 random ones."""
+    w = wl.binary32_bert()
+    ranges = sample_columns(w.d, 1024, 1031, 32, seed=5)
+    ex, em = _run_both(w, w.steps, w.mode, optimizer, ranges=ranges)
+    assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("shape,n,d", [("chain", 8, 1024), ("star", 12, 515), ("binary", 31, 257),
+                                       ("random", 20, 333), ("pair", 2, 64)])
+def test_lost_messages_every_coordinate(shape, n, d, mode):
+    """Every step loses each message with probability 0.15 (masks seeded and
+    shared with the oracle); counters bit-exact, models within tolerance."""
+    edges = {"chain": wl.chain(n), "star": wl.star(n), "binary": wl.binary_tree(n),
+             "random": wl.random_tree(n, 6), "pair": wl.chain(2)}[shape]
+    w = wl.Workload(shape, n, edges, d, wl.identity_mix(n), 1.0, 0.1, 0.1, 0.1, 30)
+    lost = (np.random.default_rng(n).random((w.steps, w.E)) < 0.15).astype(np.uint8)
+    ex, em = _run_both(w, w.steps, mode, lost=lost)
+    assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+def test_lost_messages_with_momentum_full_size_sampled():
+    """Section 4.4's setting, synthetically: 16 workers on a binary tree,
+    VGG-11-sized vector, Nesterov momentum, 10 % of messages lost, robust
+    rebuild; 60 steps."""
+    w = wl.Workload("binary16_d9231114", 16, wl.binary_tree(16), 9_231_114, wl.identity_mix(16),
+                    1.0, 0.05, 0.05, 0.0, 60)
+    lost = (np.random.default_rng(7).random((w.steps, w.E)) < 0.10).astype(np.uint8)
+    ranges = sample_columns(w.d, 1024, 1031, 32, seed=6)
+    ex, em = _run_both(w, w.steps, 1, "nesterov", lost=lost, ranges=ranges)
+    assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+def test_relay_init_zeroes_optimizer_state():
+    run = rs.RelayRun(3, 100, wl.chain(3), device="cuda:0", optimizer=("adam", 0.9, 0.99, 1e-8))
+    for t in run.state:
+        t.fill_(7.0)
+    run.init(0.0, 0, wl.identity_mix(3), 1.0, 0, 0.1)
+    torch.cuda.synchronize()
+    for t in run.state:
+        assert torch.all(t[:, :100] == 0)

@@ -95,15 +95,16 @@ def test_counts_bit_exact_all_small_trees(n):
 
 @pytest.mark.parametrize("w", wl.all_workloads(), ids=lambda w: w.name)
 def test_counts_bit_exact_workload_trees(w):
-    h = rs.relay_create(w.n, 0, w.edges)
-    counts = torch.zeros(w.E, dtype=torch.int32, device="cuda:0")
-    want = np.zeros(w.E, dtype=np.int32)
-    steps = tu.diameter(w.n, w.edges.tolist()) + 3
-    for t in range(steps):
-        rs.relay_step_counts(h, counts)
-    oracle.run(w.n, w.edges, np.zeros((w.n, 0)), np.zeros((w.n, 0)), np.zeros((w.E, 0)), want, 0,
-               0, 0, 0, steps, 0)
-    assert np.array_equal(counts.cpu().numpy(), want)
+    for edges in (w.edges if isinstance(w.edges, list) else [w.edges]):
+        h = rs.relay_create(w.n, 0, edges)
+        counts = torch.zeros(w.E, dtype=torch.int32, device="cuda:0")
+        want = np.zeros(w.E, dtype=np.int32)
+        steps = tu.diameter(w.n, edges.tolist()) + 3
+        for t in range(steps):
+            rs.relay_step_counts(h, counts)
+        oracle.run(w.n, edges, np.zeros((w.n, 0)), np.zeros((w.n, 0)), np.zeros((w.E, 0)), want,
+                   0, 0, 0, 0, steps, 0)
+        assert np.array_equal(counts.cpu().numpy(), want)
 
 
 # ------------------------------------------------------- full-vector parity
@@ -199,7 +200,8 @@ def test_deterministic_and_resumable():
     for _ in range(10):
         b.step(w.lr, w.seed)
     torch.cuda.synchronize()
-    assert torch.equal(a.x, b.x) and torch.equal(a.messages, b.messages)
+    assert torch.equal(a.x[:, :w.d], b.x[:, :w.d])
+    assert torch.equal(a.messages[:, :w.d], b.messages[:, :w.d])
     assert torch.equal(a.counts, b.counts)
 
 

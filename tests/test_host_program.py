@@ -28,8 +28,10 @@ def _built():
 REG_DEG = 4
 
 
-def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0=0):
-    """One step executed the way relay_counts_kernel + relay_models_kernel do."""
+def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0=0, lost=None):
+    """One step executed the way relay_counts_kernel + relay_models_kernel do
+    (lost: E flags of messages lost in transit, or None)."""
+    lost = np.zeros(2 * (n - 1), dtype=bool) if lost is None else np.asarray(lost, dtype=bool)
     nslots, order, node, pos = rs.relay_program(h)
     E = 2 * (n - 1)
     src, dst = rs.relay_edges(h)
@@ -37,8 +39,8 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
     counts = np.zeros(E, dtype=np.int32)
     for e in range(E):
         deg, pb = node[src[e]][0], node[src[e]][1]
-        counts[e] = 1 + sum(counts_old[pos[pb + s][0]] for s in range(deg)
-                            if pos[pb + s][0] != (e ^ 1))
+        counts[e] = 0 if lost[e] else 1 + sum(counts_old[pos[pb + s][0]] for s in range(deg)
+                                              if pos[pb + s][0] != (e ^ 1))
     nbar = [1 + sum(counts[pos[node[i][1] + s][0]] for s in range(node[i][0])) for i in range(n)]
     if mode == 0:
         scale = [1.0 / nb for nb in nbar]
@@ -88,6 +90,7 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
                 # the parent is wide: recv holds its total, which stays live
                 assert slots[recv] is not None
                 m = slots[recv] - msg_in[pos[pb + ppos][1]]
+                m = 0 * m if lost[pos[pb + ppos][0]] else m
                 msg_out[pos[pb + ppos][0]] = m
                 acc = acc + m
             else:
@@ -96,6 +99,7 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
             m = [msg_in[pos[pb + s][0]] for s in range(deg)]
             for s in range(deg):
                 out = xh + sum((m[r] for r in range(deg) if r != s), np.zeros(L))
+                out = 0 * out if lost[pos[pb + s][1]] else out
                 msg_out[pos[pb + s][1]] = out
                 if s == ppos:
                     to_parent(rec, out)
@@ -105,6 +109,7 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
             total = xh + sum(msg_in[pos[pb + s][0]] for s in range(deg))
             if ppos >= 0:
                 out = total - msg_in[pos[pb + ppos][0]]
+                out = 0 * out if lost[pos[pb + ppos][1]] else out
                 msg_out[pos[pb + ppos][1]] = out
                 to_parent(rec, out)
             write(tot, total)
@@ -117,8 +122,9 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
     return xnew, msg_out, counts, nslots
 
 
-def check_tree(n, edges, mode, steps=3, L=3, seed=1):
+def check_tree(n, edges, mode, steps=3, L=3, seed=1, p_lost=0.0):
     h = rs.relay_create(n, L, edges)
+    lost_rng = np.random.default_rng(1000 + n)
     rng = np.random.default_rng(n)
     mu = rng.normal(size=(n, L))
     x = np.tile(rng.normal(size=L), (n, 1))
@@ -129,8 +135,10 @@ def check_tree(n, edges, mode, steps=3, L=3, seed=1):
     msg = np.zeros((E, L))
     counts = np.zeros(E, dtype=np.int32)
     for t in range(steps):
-        x, msg, counts, nslots = run_program(h, n, x, mu, msg, counts, 0.3, 0.2, seed, t, mode)
-        st.advance(1, 0.3, 0.2, seed, mode)
+        lost = (lost_rng.random(E) < p_lost).astype(np.uint8)
+        x, msg, counts, nslots = run_program(h, n, x, mu, msg, counts, 0.3, 0.2, seed, t, mode,
+                                             lost=lost)
+        st.advance(1, 0.3, 0.2, seed, mode, drop=lost[None, :] if p_lost > 0 else None)
         assert np.array_equal(counts, st.counts)
         assert np.allclose(x, st.x, rtol=1e-12, atol=1e-12)
         assert np.allclose(msg, st.msg, rtol=1e-12, atol=1e-12)
@@ -157,6 +165,18 @@ def test_program_matches_oracle_workload_trees(shape, mode):
     edges = trees[shape]
     n = int(edges.max()) + 1
     check_tree(n, edges, mode, steps=2, L=2)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("shape", ["star", "binary", "random40", "star9", "chain"])
+def test_program_with_lost_messages_matches_oracle(shape, mode):
+    """Lost messages (Section 4.4) are zeroed where the kernel zeroes them --
+    including the messages a wide node's children form from its total."""
+    trees = {"star": wl.star(20), "binary": wl.binary_tree(31), "random40": wl.random_tree(40, 9),
+             "star9": wl.star(9, hub=4), "chain": wl.chain(12)}
+    edges = trees[shape]
+    n = int(edges.max()) + 1
+    check_tree(n, edges, mode, steps=6, L=2, p_lost=0.25)
 
 
 def test_slot_counts_of_workload_trees():
