@@ -223,7 +223,7 @@ def run_reference(args, w, rank: int):
     print(json.dumps(line), flush=True)
 
 
-def workload_config(w, gpus: int) -> dict:
+def workload_config(w, gpus: int, args=None) -> dict:
     shape = {"binary": "balanced binary tree (heap order)", "chain": "chain", "star": "star",
              "torus": "uniform spanning tree of the 8x8 torus",
              "double": "double binary trees (two complementary trees, half the coordinates each)"}
@@ -233,7 +233,9 @@ def workload_config(w, gpus: int) -> dict:
             "sigma": w.sigma, "lr": w.lr, "objective": "identity-Hessian heterogeneous quadratics",
             "l2": f"inputs larger than L2 ({w.bytes_per_step() / 1e9:.1f} GB moved per step)",
             "parallelism": f"d-sharded over {gpus} rank(s), no collective" if gpus > 1
-            else "1 GPU"}
+            else "1 GPU",
+            **({"algorithm": args.algorithm, "local_optimizer": args.optimizer,
+                "lost_prob": args.lost_prob, "mu": args.objective} if args is not None else {})}
 
 
 # ------------------------------------------------------------------ native
@@ -249,12 +251,18 @@ def run_native(args, w, rank: int, world: int):
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
     c0 = shard_offset(rank, w.d)
-    run = rs.RelayRun(w.n, w.d, w.edges, device=dev, mode=w.mode, c0=c0, objective=args.objective)
+    optimizer = {"sgd": None, "nesterov": ("nesterov", 0.9),
+                 "adam": ("adam", 0.9, 0.999, 1e-8)}[args.optimizer]
+    run = rs.RelayRun(w.n, w.d, w.edges, device=dev, mode=w.mode, c0=c0, objective=args.objective,
+                      optimizer=optimizer, algorithm=args.algorithm)
+    lost_rng = np.random.default_rng(1234 + rank)
     run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
     h = run.h
 
     def one_step(ev=None):
         for k, tr in enumerate(run.trees):
+            if args.lost_prob > 0:  # messages lost in transit this step (Section 4.4)
+                rs.relay_set_lost_messages(tr.h, lost_rng.random(tr.E) < args.lost_prob)
             if ev is not None:
                 ev[k][0].record(stream)
             rs.relay_step_counts(tr.h, tr.counts, stream)
@@ -300,13 +308,15 @@ def run_native(args, w, rank: int, world: int):
     peak_src = "measured" if peak else "fallback"
     peak = peak or FALLBACK_HBM_GBS
     mean_models_ms = statistics.mean(models_ms)
-    alg_bytes = w.bytes_per_step()
-    moved = alg_bytes if args.objective == "generated" else w.bytes_per_step_with_mu()
+    state_rows = {"sgd": 0, "nesterov": 2, "adam": 4}[args.optimizer]  # optimiser state read+write
+    alg_bytes = w.bytes_per_step() + 4 * w.d * w.n * state_rows
+    moved = alg_bytes if args.objective == "generated" else alg_bytes + 4 * w.d * w.n
     achieved = alg_bytes / (mean_models_ms / 1e3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4), "traffic": traffic_per_launch(w, args.objective),
                 "kernel": "relay_models_kernel", "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": alg_bytes,
+                "algorithmic_bytes_rule": "4 d (2n + 2E) [+ 4 d n x optimiser-state rows]",
                 "objective": args.objective,
                 "design_bytes_per_launch": moved,
                 "achieved_design_bytes": round(moved / (mean_models_ms / 1e3) / 1e9, 1),
@@ -319,7 +329,7 @@ def run_native(args, w, rank: int, world: int):
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": workload_config(w, world), "roofline": roofline, "cpu_baseline": cpu,
+            "config": workload_config(w, world, args), "roofline": roofline, "cpu_baseline": cpu,
             "e2e": e2e, "gpu_launches": 2 * T * args.steps, "clocks": clocks.summary(),
             "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1)}
     print(json.dumps(line), flush=True)
@@ -419,6 +429,12 @@ def main(argv=None):
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     p.add_argument("--e2e-steps", type=int, default=3)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--optimizer", choices=["sgd", "nesterov", "adam"], default="sgd",
+                   help="local optimiser of the local step (appendix: momentum / Adam)")
+    p.add_argument("--algorithm", choices=["relaysgd", "grad", "dme"], default="relaysgd",
+                   help="Algorithm 1 (default), 6 (relayed updates) or 5 (mean estimation)")
+    p.add_argument("--lost-prob", type=float, default=0.0,
+                   help="probability that each message is lost in transit, per step")
     p.add_argument("--objective", choices=["generated", "stored"], default="stored",
                    help="regenerate the centres mu in the kernel, or read a stored mu array")
     p.add_argument("--d", type=int, default=None,

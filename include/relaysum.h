@@ -106,6 +106,19 @@ int relay_set_strides(relay_handle *h, int64_t ld_x, int64_t ld_msg);
 int relay_set_local_optimizer(relay_handle *h, int32_t kind, float beta1, float beta2, float eps,
                               float *state1, float *state2);
 
+#define RELAY_ALGO_RELAYSGD 0  /* Algorithm 1: x' = rebuild of x^{t+1/2} and the messages      */
+#define RELAY_ALGO_GRAD 1      /* Algorithm 6: relay the update u; x' = x + (u + sum m) / n    */
+#define RELAY_ALGO_DME 2       /* Algorithm 5: relay samples mu + sigma xi; x holds y += ...  */
+
+/* Which algorithm runs on the relay (appendix "RelaySum for distributed mean
+ * estimation", "Alternative optimizer based on RelaySum").  For RELAY_ALGO_DME
+ * x holds the running sums y_i, the samples are mu_i + sigma xi_i^t (the
+ * objective's centres and noise), and dme_count (device int64 [n], zeroed by
+ * relay_init) accumulates s_i += 1 + sum_j c^t_{j->i} at every step; the
+ * estimate of worker i is y_i / s_i.  RELAY_ALGO_GRAD needs no counters (they
+ * are still maintained).  Default RELAY_ALGO_RELAYSGD. */
+int relay_set_algorithm(relay_handle *h, int32_t algo, int64_t *dme_count);
+
 /* Messages lost in transit (Section 4.4, "Robustness to unreliable
  * communication"): host uint8 [E], non-zero = the message sent on that
  * directed edge by every later step never arrives, so its receiver reads

@@ -86,7 +86,11 @@ def _load():
 
 class _Opts(ctypes.Structure):
     _fields_ = [("opt", ctypes.c_int), ("beta1", ctypes.c_double), ("beta2", ctypes.c_double),
-                ("eps", ctypes.c_double), ("drop", ctypes.POINTER(ctypes.c_uint8))]
+                ("eps", ctypes.c_double), ("drop", ctypes.POINTER(ctypes.c_uint8)),
+                ("algo", ctypes.c_int), ("dme_count", ctypes.POINTER(ctypes.c_int64))]
+
+
+ALGO_RELAYSGD, ALGO_GRAD, ALGO_DME = 0, 1, 2
 
 
 OPT_SGD, OPT_NESTEROV, OPT_ADAM = 0, 1, 2
@@ -195,7 +199,7 @@ def run(n: int, edge_list, x: np.ndarray, mu: np.ndarray, msg: np.ndarray, count
 def run_ext(n: int, edge_list, x, mu, msg, counts, lr: float, sigma: float, seed: int,
             step0: int, steps: int, mode: int = 0, c0: int = 0, opt: int = OPT_SGD,
             beta1: float = 0.0, beta2: float = 0.0, eps: float = 0.0, s1=None, s2=None,
-            drop=None):
+            drop=None, algo: int = ALGO_RELAYSGD, dme_count=None):
     """run() with a local optimiser (SGD / Nesterov momentum / Adam, state
     arrays s1, s2 [n][len] in place) and an optional mask drop[steps][E] of
     lost messages."""
@@ -209,7 +213,10 @@ def run_ext(n: int, edge_list, x, mu, msg, counts, lr: float, sigma: float, seed
         if a is not None:
             assert a.dtype == np.float64 and a.flags.c_contiguous and a.shape == (n, length)
     assert counts.dtype == np.int32 and counts.shape == (E,)
-    o = _Opts(opt, beta1, beta2, eps, None)
+    o = _Opts(opt, beta1, beta2, eps, None, algo, None)
+    if algo == ALGO_DME:
+        assert dme_count is not None and dme_count.dtype == np.int64 and dme_count.shape == (n,)
+        o.dme_count = dme_count.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))
     if drop is not None:
         drop = np.ascontiguousarray(np.asarray(drop, dtype=np.uint8).reshape(steps, E))
         o.drop = drop.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8))
@@ -251,11 +258,14 @@ class State:
         self.step = 0
         self.s1 = np.zeros((self.n, self.length))
         self.s2 = np.zeros((self.n, self.length))
+        self.dme_count = np.zeros(self.n, dtype=np.int64)
 
     def advance(self, steps: int, lr: float, sigma: float, seed: int, mode: int = 0,
                 opt: int = OPT_SGD, beta1: float = 0.0, beta2: float = 0.0, eps: float = 0.0,
-                drop=None):
-        if opt == OPT_SGD and drop is None:
+                drop=None, algo: int = ALGO_RELAYSGD):
+        if not hasattr(self, "dme_count"):
+            self.dme_count = np.zeros(self.n, dtype=np.int64)
+        if opt == OPT_SGD and drop is None and algo == ALGO_RELAYSGD:
             nbar = run(self.n, self.edges, self.x, self.mu, self.msg, self.counts, lr, sigma,
                        seed, self.step, steps, mode, self.c0)
         else:
@@ -264,6 +274,6 @@ class State:
                 self.s2 = np.zeros((self.n, self.length))
             nbar = run_ext(self.n, self.edges, self.x, self.mu, self.msg, self.counts, lr, sigma,
                            seed, self.step, steps, mode, self.c0, opt, beta1, beta2, eps,
-                           self.s1, self.s2, drop)
+                           self.s1, self.s2, drop, algo, self.dme_count)
         self.step += steps
         return nbar

@@ -252,16 +252,32 @@ typedef struct {
     int opt;
     double beta1, beta2, eps;
     const uint8_t *drop;  /* [steps][E] or NULL */
+    int algo;             /* 0 RelaySGD (Alg. 1), 1 RelaySum/Grad (Alg. 6), 2 DME (Alg. 5) */
+    int64_t *dme_count;   /* algo 2: s_i, [n], in/out */
 } oracle_opts;
+
+/* The two other algorithms of the appendix on the same relay mechanism:
+ *
+ *   RelaySum/Grad (Algorithm 6): the relayed value is the update
+ *     u_i^t = x_i^{t+1/2} - x_i^t (= -lr g for SGD) and
+ *     x_i^{t+1} = x_i^t + (u_i^t + sum_j m^t_{j->i}) / n      (no counters used)
+ *
+ *   RelaySum for distributed mean estimation (Algorithm 5): the relayed value
+ *     is a sample dhat_i^t = mu_i + sigma xi_i^t; x holds the running sum y and
+ *     y_i^{t+1} = y_i^t + dhat_i^t + sum_j m^t_{j->i},
+ *     s_i^{t+1} = s_i^t + 1 + sum_j c^t_{j->i}   (dme_count),
+ *   the estimate of worker i being y_i / s_i. */
 
 int oracle_run_ext(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t len,
                    double *x, const double *mu, double *msg, int32_t *counts, double *s1,
                    double *s2, double lr, double sigma, uint64_t seed, int64_t step0,
                    int64_t steps, int mode, const oracle_opts *opts, int32_t *nbar) {
     const int opt = opts ? opts->opt : 0;
+    const int algo = opts ? opts->algo : 0;
     if (len < 0 || c0 < 0 || step0 < 0 || steps < 0 || (mode != 0 && mode != 1) || opt < 0 ||
-        opt > 2)
+        opt > 2 || algo < 0 || algo > 2)
         return ORACLE_EINVAL;
+    if (algo == 2 && !opts->dme_count) return ORACLE_EINVAL;
     if ((opt >= 1 && !s1) || (opt == 2 && !s2)) return ORACLE_EINVAL;
     if (step0 + steps > 4294967296LL) return ORACLE_EINVAL;
     otree t;
@@ -292,8 +308,9 @@ int oracle_run_ext(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t
             int32_t s = 1;
             for (int k = t.nbr_off[i]; k < t.nbr_off[i + 1]; ++k) s += counts[t.in_edge[k]];
             nb[i] = s;
+            if (algo == 2) opts->dme_count[i] += s;
         }
-        /* local step */
+        /* local step (xh holds the relayed value: x^{t+1/2}, u or dhat) */
         const double k_adam = (double)(t_step + 1);
         for (int i = 0; i < n; ++i)
             for (int64_t c = 0; c < len; ++c) {
@@ -301,6 +318,10 @@ int oracle_run_ext(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t
                 double xv = x[ic];
                 double xi = oracle_normal(seed, c0 + c, (uint32_t)i, (uint32_t)t_step, 0u);
                 double g = (xv - mu[ic]) + sigma * xi;
+                if (algo == 2) {
+                    xh[ic] = mu[ic] + sigma * xi;  /* the sample dhat_i^t */
+                    continue;
+                }
                 if (opt == 0) {
                     xh[ic] = xv - lr * g;
                 } else if (opt == 1) {
@@ -314,6 +335,7 @@ int oracle_run_ext(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t
                     const double denom = sqrt(s2[ic]) / sqrt(bc2) + opts->eps;
                     xh[ic] = xv - (lr / bc1) * s1[ic] / denom;
                 }
+                if (algo == 1) xh[ic] -= xv;  /* the update u = x^{t+1/2} - x^t */
             }
         /* relay messages m^{t} from x^{t+1/2} and m^{t-1} */
         for (int e = 0; e < E; ++e) {
@@ -331,7 +353,11 @@ int oracle_run_ext(int n, const int32_t *edges, int n_edges, int64_t c0, int64_t
                 double s = xh[(int64_t)i * len + c];
                 for (int k = t.nbr_off[i]; k < t.nbr_off[i + 1]; ++k)
                     s += m_new[(int64_t)t.in_edge[k] * len + c];
-                if (mode == 0) {
+                if (algo == 1) {
+                    x[(int64_t)i * len + c] += s / (double)n;
+                } else if (algo == 2) {
+                    x[(int64_t)i * len + c] += s;
+                } else if (mode == 0) {
                     x[(int64_t)i * len + c] = s / (double)nb[i];
                 } else {
                     double xold = x[(int64_t)i * len + c];

@@ -14,22 +14,24 @@ steps.
 from __future__ import annotations
 
 from ._native import (RELAY_EINVAL, RELAY_ECUDA, RELAY_ENOMEM, RELAY_ENOTTREE, RELAY_EUNSUPPORTED,
-                      RELAY_MAX_N, RELAY_OK, RELAY_OPT_ADAM, RELAY_OPT_NESTEROV, RELAY_OPT_SGD,
+                      RELAY_ALGO_DME, RELAY_ALGO_GRAD, RELAY_ALGO_RELAYSGD, RELAY_MAX_N, RELAY_OK,
+                      RELAY_OPT_ADAM, RELAY_OPT_NESTEROV, RELAY_OPT_SGD,
                       RelayError, RelayHandle, RelayRun, library_path,
                       relay_create, relay_destroy, relay_edges, relay_error_string,
                       relay_fill_objective, relay_init, relay_ld, relay_nbar, relay_num_edges,
                       relay_program, relay_set_coord_offset, relay_set_objective,
-                      relay_set_local_optimizer, relay_set_lost_messages,
+                      relay_set_algorithm, relay_set_local_optimizer, relay_set_lost_messages,
                       relay_set_objective_generated, relay_set_rebuild_mode, relay_set_strides,
                       relay_step,
                       relay_step_counts, relay_step_models)
 
 __all__ = [
     "RELAY_OK", "RELAY_EINVAL", "RELAY_ENOTTREE", "RELAY_ECUDA", "RELAY_ENOMEM",
-    "RELAY_EUNSUPPORTED", "RELAY_MAX_N", "RELAY_OPT_SGD", "RELAY_OPT_NESTEROV", "RELAY_OPT_ADAM", "RelayError", "RelayHandle", "RelayRun", "library_path",
+    "RELAY_EUNSUPPORTED", "RELAY_MAX_N", "RELAY_OPT_SGD", "RELAY_OPT_NESTEROV", "RELAY_OPT_ADAM",
+    "RELAY_ALGO_RELAYSGD", "RELAY_ALGO_GRAD", "RELAY_ALGO_DME", "RelayError", "RelayHandle", "RelayRun", "library_path",
     "relay_create", "relay_destroy", "relay_ld", "relay_num_edges", "relay_edges",
     "relay_set_rebuild_mode", "relay_set_strides", "relay_set_local_optimizer",
-    "relay_set_lost_messages", "relay_set_coord_offset", "relay_set_objective",
+    "relay_set_lost_messages", "relay_set_algorithm", "relay_set_coord_offset", "relay_set_objective",
     "relay_set_objective_generated", "relay_fill_objective", "relay_init", "relay_step_counts",
     "relay_step_models", "relay_step",
     "relay_nbar", "relay_program", "relay_error_string",

@@ -19,6 +19,9 @@ RELAY_MAX_N = 256
 RELAY_OPT_SGD = 0
 RELAY_OPT_NESTEROV = 1
 RELAY_OPT_ADAM = 2
+RELAY_ALGO_RELAYSGD = 0
+RELAY_ALGO_GRAD = 1
+RELAY_ALGO_DME = 2
 
 _lock = threading.Lock()
 _lib = None
@@ -50,6 +53,7 @@ def _load():
             "relay_set_strides": (ctypes.c_int, [vp, i64, i64]),
             "relay_set_local_optimizer": (ctypes.c_int, [vp, i32, f32, f32, f32, vp, vp]),
             "relay_set_lost_messages": (ctypes.c_int, [vp, vp]),
+            "relay_set_algorithm": (ctypes.c_int, [vp, i32, vp]),
             "relay_set_coord_offset": (ctypes.c_int, [vp, i64]),
             "relay_set_objective": (ctypes.c_int, [vp, vp, f32]),
             "relay_set_objective_generated": (ctypes.c_int, [vp, vp, i32, f32, u64, f32]),
@@ -181,6 +185,10 @@ def relay_set_local_optimizer(h, kind: int, beta1: float = 0.0, beta2: float = 0
            "relay_set_local_optimizer")
 
 
+def relay_set_algorithm(h, algo: int, dme_count=None):
+    _check(_load().relay_set_algorithm(_h(h), int(algo), _ptr(dme_count)), "relay_set_algorithm")
+
+
 def relay_set_lost_messages(h, lost=None):
     """lost: host array of E flags (non-zero = lost) or None."""
     if lost is None:
@@ -286,8 +294,10 @@ class RelayRun:
     """
 
     def __init__(self, n: int, d: int, edges, device="cuda", mode: int = 1, c0: int = 0,
-                 objective: str = "stored", optimizer=None):
-        """optimizer: None (SGD), ("nesterov", beta1) or ("adam", beta1, beta2, eps)."""
+                 objective: str = "stored", optimizer=None, algorithm: str = "relaysgd"):
+        """optimizer: None (SGD), ("nesterov", beta1) or ("adam", beta1, beta2, eps);
+        algorithm: "relaysgd" (Alg. 1), "grad" (Alg. 6) or "dme" (Alg. 5, x holds
+        the running sums y and `dme_count` the counts s of each tree)."""
         import torch
         if objective not in ("stored", "generated"):
             raise ValueError(objective)
@@ -317,10 +327,17 @@ class RelayRun:
                 hyper = list(optimizer[1:]) + [0.0] * (3 - len(optimizer[1:]))
                 st = [_window_ptr(t, col0) if dk > 0 else None for t in self.state] + [None]
                 relay_set_local_optimizer(h, kind, hyper[0], hyper[1], hyper[2], st[0], st[1])
+            algo = {"relaysgd": RELAY_ALGO_RELAYSGD, "grad": RELAY_ALGO_GRAD,
+                    "dme": RELAY_ALGO_DME}[algorithm]
+            dme_count = (torch.zeros(n, dtype=torch.int64, device=self.device)
+                         if algo == RELAY_ALGO_DME else None)
+            relay_set_algorithm(h, algo, dme_count)
             E = relay_num_edges(h)
             msg = [torch.empty(max(E, 1), max(ld_m, 1), **f32) for _ in range(2)]
             counts = torch.zeros(max(E, 1), dtype=torch.int32, device=self.device)
-            self.trees.append(_TreeState(h, col0, dk, E, msg, counts))
+            tr = _TreeState(h, col0, dk, E, msg, counts)
+            tr.dme_count = dme_count
+            self.trees.append(tr)
         self.t = 0
 
     # single-tree conveniences

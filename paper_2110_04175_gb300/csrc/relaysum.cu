@@ -49,6 +49,9 @@ struct relay_handle {
     float beta1 = 0.0f, beta2 = 0.0f, eps = 0.0f;
     float* s1 = nullptr;  // momentum buffer / Adam first moment, [n][ld_x]
     float* s2 = nullptr;  // Adam second moment, [n][ld_x]
+    // algorithm on the relay: 0 RelaySGD (Alg. 1), 1 RelaySum/Grad (Alg. 6), 2 DME (Alg. 5)
+    int32_t algo = 0;
+    int64_t* dme_count = nullptr;  // algo 2: s_i, device int64 [n]
     // messages lost in transit (Section 4.4), one bit per directed edge
     bool has_lost = false;
     uint32_t lost[relaysum::kMaxE / 32 + 1] = {};
@@ -168,13 +171,15 @@ __device__ __forceinline__ void st_stream(float* p, float4 v) {
 
 // c^t_{i->j} = 1 + sum_{k in N(i)\j} c^{t-1}_{k->i}: the incoming edge from
 // j is e ^ 1 for e = i -> j.  A lost message (Section 4.4) arrives as c = 0.
+// For distributed mean estimation (Alg. 5) it also adds each worker's
+// models-received count 1 + sum_j c^t_{j->i} to the running count s_i.
 struct LostMask {
     uint32_t w[relaysum::kMaxE / 32 + 1];
     __host__ __device__ __forceinline__ bool operator()(int e) const { return (w[e >> 5] >> (e & 31)) & 1u; }
 };
 
 __global__ void relay_counts_kernel(const __grid_constant__ Program prog, const __grid_constant__ LostMask lost,
-                                    int has_lost, int32_t* counts) {
+                                    int has_lost, int32_t* counts, int64_t* dme_count) {
     __shared__ int32_t c_old[kMaxE];
     const int E = prog.E;
     for (int e = threadIdx.x; e < E; e += blockDim.x) c_old[e] = counts[e];
@@ -187,6 +192,15 @@ __global__ void relay_counts_kernel(const __grid_constant__ Program prog, const 
             if (in != (e ^ 1)) s += c_old[in];
         }
         counts[e] = (has_lost && lost(e)) ? 0 : s;  // a lost message carries no count
+    }
+    if (dme_count) {  // Alg. 5: s_i += 1 + sum_j c^t_{j->i}
+        __syncthreads();
+        for (int i = threadIdx.x; i < prog.n; i += blockDim.x) {
+            const NodeRec r = prog.node[i];
+            int64_t nb = 1;
+            for (int p = 0; p < r.deg; ++p) nb += counts[prog.pos_in[r.pos_base + p]];
+            dme_count[i] += nb;
+        }
     }
 }
 
@@ -205,6 +219,7 @@ struct ModelArgs {
     uint32_t step;
     float lr, sigma;
     int mode;         // 0: Alg. 1 rebuild, 1: robust rebuild
+    int algo;         // 0 RelaySGD, 1 RelaySum/Grad, 2 mean estimation
     int has_lost;     // any bit of `lost` set
     LostMask lost;    // messages lost in transit this step
     float* s1;        // optimiser state (momentum / Adam m), [n][ld_x]
@@ -294,25 +309,22 @@ __device__ __noinline__ void visit_wide(const Program& prog, const NodeRec& r, c
     sl[r.tot_slot] = total;
 }
 
-// Alg. 1's local step with the chosen optimiser, per coordinate.
-//   SGD:      x - lr g
-//   Nesterov: m = beta1 m + g;  x - lr (g + beta1 m)          (state s1 = m)
+// The local optimiser's update u (Alg. 1's local step is x^{t+1/2} = x + u):
+//   SGD:      u = -lr g
+//   Nesterov: m = beta1 m + g;  u = -lr (g + beta1 m)          (state s1 = m)
 //   Adam:     m = beta1 m + (1 - beta1) g;  v = beta2 v + (1 - beta2) g^2;
-//             x - adam_step m / (sqrt(v) adam_ibc2 + eps)     (s1 = m, s2 = v)
-__device__ __forceinline__ float sgd1(float lr, float x, float g) { return fmaf(-lr, g, x); }
-
+//             u = -adam_step m / (sqrt(v) adam_ibc2 + eps)     (s1 = m, s2 = v)
 template <int OPT>
-__device__ __forceinline__ float4 local_step(const ModelArgs& a, int i, int64_t q, float4 x, float4 g) {
-    if (OPT == 0) return make_float4(sgd1(a.lr, x.x, g.x), sgd1(a.lr, x.y, g.y), sgd1(a.lr, x.z, g.z),
-                                     sgd1(a.lr, x.w, g.w));
+__device__ __forceinline__ float4 local_update(const ModelArgs& a, int i, int64_t q, float4 g) {
+    if (OPT == 0) return scale4(g, -a.lr);
     float4* pm = reinterpret_cast<float4*>(a.s1 + i * a.ld_x + 4 * q);
     float4 m = *pm;
     if (OPT == 1) {
         m = make_float4(fmaf(a.beta1, m.x, g.x), fmaf(a.beta1, m.y, g.y), fmaf(a.beta1, m.z, g.z),
                         fmaf(a.beta1, m.w, g.w));
         __stcs(pm, m);
-        return make_float4(fmaf(-a.lr, fmaf(a.beta1, m.x, g.x), x.x), fmaf(-a.lr, fmaf(a.beta1, m.y, g.y), x.y),
-                           fmaf(-a.lr, fmaf(a.beta1, m.z, g.z), x.z), fmaf(-a.lr, fmaf(a.beta1, m.w, g.w), x.w));
+        return make_float4(-a.lr * fmaf(a.beta1, m.x, g.x), -a.lr * fmaf(a.beta1, m.y, g.y),
+                           -a.lr * fmaf(a.beta1, m.z, g.z), -a.lr * fmaf(a.beta1, m.w, g.w));
     }
     float4* pv = reinterpret_cast<float4*>(a.s2 + i * a.ld_x + 4 * q);
     float4 v = *pv;
@@ -323,10 +335,8 @@ __device__ __forceinline__ float4 local_step(const ModelArgs& a, int i, int64_t 
                     fmaf(a.beta2, v.z, c2 * g.z * g.z), fmaf(a.beta2, v.w, c2 * g.w * g.w));
     __stcs(pm, m);
     __stcs(pv, v);
-    auto upd = [&](float xx, float mm, float vv) {
-        return xx - a.adam_step * mm / fmaf(sqrtf(vv), a.adam_ibc2, a.eps);
-    };
-    return make_float4(upd(x.x, m.x, v.x), upd(x.y, m.y, v.y), upd(x.z, m.z, v.z), upd(x.w, m.w, v.w));
+    auto upd = [&](float mm, float vv) { return -a.adam_step * mm / fmaf(sqrtf(vv), a.adam_ibc2, a.eps); };
+    return make_float4(upd(m.x, v.x), upd(m.y, v.y), upd(m.z, v.z), upd(m.w, v.w));
 }
 
 // mu_i for quad q: read, or regenerated exactly as relay_fill_mu_kernel
@@ -362,7 +372,13 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
         const NodeRec r = prog.node[i];
         int nbar = 1;
         for (int p = 0; p < r.deg; ++p) nbar += __ldg(a.counts + prog.pos_in[r.pos_base + p]);
-        if (a.mode == 0) {
+        if (a.algo == 1) {  // x' = x + (u + sum m) / n
+            s_scale[i] = 1.0f / static_cast<float>(n);
+            s_fill[i] = static_cast<float>(n);
+        } else if (a.algo == 2) {  // y' = y + dhat + sum m
+            s_scale[i] = 1.0f;
+            s_fill[i] = 1.0f;
+        } else if (a.mode == 0) {
             s_scale[i] = 1.0f / static_cast<float>(nbar);
             s_fill[i] = 0.0f;
         } else {
@@ -388,12 +404,23 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
             const float4 mv = centre<OBJ>(obj, mu_key, a, i, q, cen, static_cast<int>(blockDim.x));
             const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i),
                                      a.step, 0u, a.key);
-            // g = (x - mu) + sigma * xi, then the local optimiser's x^{t+1/2}
-            const float4 g = make_float4(fmaf(a.sigma, z.x, xv.x - mv.x), fmaf(a.sigma, z.y, xv.y - mv.y),
-                                         fmaf(a.sigma, z.z, xv.z - mv.z), fmaf(a.sigma, z.w, xv.w - mv.w));
-            const float4 xh = local_step<OPT>(a, i, q, xv, g);
+            // the relayed value: x^{t+1/2} = x + u (Alg. 1), the update u
+            // (Alg. 6) or the sample mu + sigma xi (Alg. 5), with
+            // g = (x - mu) + sigma xi
+            float4 xh;
+            if (a.algo == 2) {
+                xh = make_float4(fmaf(a.sigma, z.x, mv.x), fmaf(a.sigma, z.y, mv.y), fmaf(a.sigma, z.z, mv.z),
+                                 fmaf(a.sigma, z.w, mv.w));
+            } else {
+                const float4 g = make_float4(fmaf(a.sigma, z.x, xv.x - mv.x), fmaf(a.sigma, z.y, xv.y - mv.y),
+                                             fmaf(a.sigma, z.z, xv.z - mv.z), fmaf(a.sigma, z.w, xv.w - mv.w));
+                const float4 u = local_update<OPT>(a, i, q, g);
+                xh = (a.algo == 1) ? u : add4(xv, u);
+            }
+            // the rebuild sum starts from fill_i x_i (robust rule: n - nbar_i;
+            // Alg. 6: n; Alg. 5: 1; Alg. 1: nothing)
             float4 acc = xh;
-            if (a.mode == 1) acc = add4(scale4(xv, s_fill[i]), xh);
+            if (s_fill[i] != 0.0f) acc = add4(scale4(xv, s_fill[i]), xh);
             if (r.recv_slot >= 0) {
                 float4 recv = sl[r.recv_slot];
                 if (r.flags & relaysum::kRecvFromTotal) {
@@ -648,6 +675,14 @@ int relay_set_local_optimizer(relay_handle* h, int32_t kind, float beta1, float 
     return RELAY_OK;
 }
 
+int relay_set_algorithm(relay_handle* h, int32_t algo, int64_t* dme_count) {
+    if (!h || algo < RELAY_ALGO_RELAYSGD || algo > RELAY_ALGO_DME) return RELAY_EINVAL;
+    if (algo == RELAY_ALGO_DME && !dme_count) return RELAY_EINVAL;
+    h->algo = algo;
+    h->dme_count = algo == RELAY_ALGO_DME ? dme_count : nullptr;
+    return RELAY_OK;
+}
+
 int relay_set_lost_messages(relay_handle* h, const uint8_t* lost) {
     if (!h) return RELAY_EINVAL;
     std::memset(h->lost, 0, sizeof(h->lost));
@@ -742,6 +777,9 @@ int relay_init(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* c
                      (msg_b && !aligned16(msg_b))))
         return RELAY_EINVAL;
     if (E > 0 && cudaMemsetAsync(counts, 0, sizeof(int32_t) * E, stream) != cudaSuccess) return RELAY_ECUDA;
+    if (h->dme_count &&
+        cudaMemsetAsync(h->dme_count, 0, sizeof(int64_t) * h->prog.n, stream) != cudaSuccess)
+        return RELAY_ECUDA;
     if (h->d == 0) return RELAY_OK;
     // optimiser state starts at zero (momentum buffer, Adam moments)
     const size_t state_bytes = static_cast<size_t>((h->prog.n - 1) * h->ld_x + 4 * h->nquads) * 4;
@@ -759,11 +797,12 @@ int relay_init(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* c
 
 int relay_step_counts(relay_handle* h, int32_t* counts, relay_stream_t stream) {
     if (!h) return RELAY_EINVAL;
-    if (h->prog.E == 0) return RELAY_OK;
-    if (!counts) return RELAY_EINVAL;
+    if (h->prog.E == 0 && h->algo != RELAY_ALGO_DME) return RELAY_OK;
+    if (!counts && h->prog.E > 0) return RELAY_EINVAL;
     LostMask lost;
     std::memcpy(lost.w, h->lost, sizeof(lost.w));
-    relay_counts_kernel<<<1, 256, 0, stream>>>(h->prog, lost, h->has_lost ? 1 : 0, counts);
+    relay_counts_kernel<<<1, 256, 0, stream>>>(h->prog, lost, h->has_lost ? 1 : 0, counts,
+                                               h->algo == RELAY_ALGO_DME ? h->dme_count : nullptr);
     return launch_status();
 }
 
@@ -788,6 +827,7 @@ int relay_step_models(relay_handle* h, float* x, const float* msg_in, float* msg
     a.lr = lr;
     a.sigma = h->sigma;
     a.mode = h->mode;
+    a.algo = h->algo;
     a.has_lost = h->has_lost ? 1 : 0;
     std::memcpy(a.lost.w, h->lost, sizeof(a.lost.w));
     a.s1 = h->s1;

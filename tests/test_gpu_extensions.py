@@ -128,3 +128,72 @@ def test_relay_init_zeroes_optimizer_state():
     torch.cuda.synchronize()
     for t in run.state:
         assert torch.all(t[:, :100] == 0)
+
+
+# ------------------------------------------------ RelaySum/Grad and DME
+
+ALGOS = {"grad": oracle.ALGO_GRAD, "dme": oracle.ALGO_DME}
+
+
+@pytest.mark.parametrize("lost_p", [0.0, 0.2])
+@pytest.mark.parametrize("algorithm", ["grad", "dme"])
+@pytest.mark.parametrize("shape,n,d", [("chain", 8, 1024), ("star", 10, 515), ("binary", 15, 517),
+                                       ("single", 1, 129), ("random", 12, 260)])
+def test_other_algorithms_every_coordinate(shape, n, d, algorithm, lost_p):
+    """Algorithm 6 (relayed updates) and Algorithm 5 (relayed samples, running
+    sums and counts) against the oracle; DME's counts s_i bit-exact."""
+    edges = {"chain": wl.chain(n), "star": wl.star(n), "binary": wl.binary_tree(n),
+             "single": np.zeros((0, 2), np.int32), "random": wl.random_tree(n, 3)}[shape]
+    w = wl.Workload(shape, n, edges, d, wl.identity_mix(n), 1.0, 0.2, 0.1, 0.1, 25)
+    E = 2 * (n - 1)
+    lost = (np.random.default_rng(n).random((w.steps, E)) < lost_p).astype(np.uint8)
+    run = rs.RelayRun(n, d, edges, device="cuda:0", algorithm=algorithm)
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    st = oracle.State(n, edges, d)
+    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+    if algorithm == "dme":
+        st.x[:] = 0.0  # running sums start at zero
+        run.x.zero_()
+    for t in range(w.steps):
+        if lost_p > 0:
+            run.set_lost(lost[t])
+        run.step(w.lr, w.seed)
+        st.advance(1, float(np.float32(w.lr)), float(np.float32(w.sigma)), w.seed, 1,
+                   drop=lost[t:t + 1] if lost_p > 0 else None, algo=ALGOS[algorithm])
+    torch.cuda.synchronize()
+    assert parity_error(run.x[:, :d].double().cpu().numpy(), st.x) <= RTOL
+    if E:
+        assert parity_error(run.messages[:E, :d].double().cpu().numpy(), st.msg) <= RTOL
+        assert np.array_equal(run.counts[:E].cpu().numpy(), st.counts)
+    if algorithm == "dme":
+        assert np.array_equal(run.trees[0].dme_count.cpu().numpy(), st.dme_count)
+
+
+@pytest.mark.parametrize("algorithm", ["grad", "dme"])
+def test_other_algorithms_full_size_sampled(algorithm):
+    """The 64-worker torus spanning tree at d = 2.5e7, 100 steps."""
+    w = wl.sweep64("torus")
+    run = rs.RelayRun(w.n, w.d, w.edges, device="cuda:0", algorithm=algorithm)
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    if algorithm == "dme":
+        run.x.zero_()
+    for _ in range(w.steps):
+        run.step(w.lr, w.seed)
+    torch.cuda.synchronize()
+    gx, ox, gm, om = [], [], [], []
+    for start, length in sample_columns(w.d, 1024, 1031, 24, seed=8):
+        st = oracle.State(w.n, w.edges, length, c0=start)
+        st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+        if algorithm == "dme":
+            st.x[:] = 0.0
+        st.advance(w.steps, float(np.float32(w.lr)), float(np.float32(w.sigma)), w.seed, 1,
+                   algo=ALGOS[algorithm])
+        gx.append(run.x[:, start:start + length].double().cpu().numpy())
+        gm.append(run.messages[:run.E, start:start + length].double().cpu().numpy())
+        ox.append(st.x)
+        om.append(st.msg)
+    assert parity_error(np.concatenate(gx, 1), np.concatenate(ox, 1)) <= RTOL
+    assert parity_error(np.concatenate(gm, 1), np.concatenate(om, 1)) <= RTOL
+    del run
+    gc.collect()
+    torch.cuda.empty_cache()

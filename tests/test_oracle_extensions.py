@@ -212,3 +212,81 @@ def test_lost_messages_equal_routing_brute_force(n, mode):
             exact = np.array([[float(v) for v in r] for r in xs[t + 1]])
             assert np.max(np.abs(st.x - exact)) <= 1e-12 * max(1.0, np.max(np.abs(exact)))
             assert list(st.counts) == cnts[t], (edges, t)
+
+
+# ------------------------------------------------ RelaySum/Grad and DME
+
+def _delays(n, edges):
+    tau = tu.distances(n, edges)
+    return [[max(tau[i][l] - 1, 0) for l in range(n)] for i in range(n)]
+
+
+@pytest.mark.parametrize("n", [1, 2, 3, 4, 5, 6])
+def test_relaysum_grad_equals_delayed_update_sums(n):
+    """Algorithm 6: every update u_l^s = -lr grad reaches every worker i, with
+    weight exactly 1/n, at step s + max(tau_il - 1, 0):
+        x_i^{t+1} = x_i^0 + 1/n sum_l sum_{s <= t - delta_il} u_l^s."""
+    rng = np.random.default_rng(50 + n)
+    trees = list(tu.all_trees(n))
+    if len(trees) > 30:
+        trees = [trees[k] for k in rng.choice(len(trees), 30, replace=False)]
+    lr = Fraction(1, 4)
+    L = 2
+    for edges in trees:
+        delta = _delays(n, edges)
+        steps = tu.diameter(n, edges) + 3
+        x0i = rng.integers(-9, 9, size=(n, L))
+        mui = rng.integers(-9, 9, size=(n, L))
+        xs = [[[Fraction(int(v)) for v in r] for r in x0i]]
+        us = []
+        for t in range(steps):
+            us.append([[-lr * (xs[t][l][c] - mui[l][c]) for c in range(L)] for l in range(n)])
+            xs.append([[xs[0][i][c] + sum(us[s][l][c] for l in range(n)
+                                          for s in range(0, t - delta[i][l] + 1)) / n
+                        for c in range(L)] for i in range(n)])
+        st = oracle.State(n, edges, L)
+        st.x, st.mu = x0i.astype(np.float64), mui.astype(np.float64)
+        for t in range(steps):
+            st.advance(1, float(lr), 0.0, 0, algo=oracle.ALGO_GRAD)
+            exact = np.array([[float(v) for v in r] for r in xs[t + 1]])
+            assert np.max(np.abs(st.x - exact)) <= 1e-12 * max(1.0, np.max(np.abs(exact))), edges
+
+
+@pytest.mark.parametrize("n", [1, 2, 3, 4, 5, 6])
+def test_dme_equals_delayed_sample_sums(n):
+    """Algorithm 5: y_i^{t+1} = sum_l sum_{s <= t - delta_il} dhat_l^s and
+    s_i^{t+1} counts those samples."""
+    rng = np.random.default_rng(60 + n)
+    trees = list(tu.all_trees(n))
+    if len(trees) > 30:
+        trees = [trees[k] for k in rng.choice(len(trees), 30, replace=False)]
+    L, sigma, seed = 3, 0.5, 21
+    for edges in trees:
+        delta = _delays(n, edges)
+        steps = tu.diameter(n, edges) + 3
+        mui = rng.integers(-5, 5, size=(n, L)).astype(np.float64)
+        samples = [[[Fraction(float(mui[l][c] + sigma * oracle.normal(seed, c, l, s, 0)))
+                     for c in range(L)] for l in range(n)] for s in range(steps)]
+        st = oracle.State(n, edges, L)
+        st.x, st.mu = np.zeros((n, L)), mui.copy()
+        for t in range(steps):
+            st.advance(1, 0.0, sigma, seed, algo=oracle.ALGO_DME)
+            y = np.array([[float(sum(samples[s][l][c] for l in range(n)
+                                     for s in range(0, t - delta[i][l] + 1))) for c in range(L)]
+                          for i in range(n)])
+            cnt = [sum(max(t - delta[i][l] + 1, 0) for l in range(n)) for i in range(n)]
+            assert np.allclose(st.x, y, rtol=1e-12, atol=1e-12), edges
+            assert list(st.dme_count) == cnt
+
+
+def test_dme_variance_shrinks_like_one_over_samples():
+    """With i.i.d. N(1, sigma^2) samples, worker i's estimate y_i / s_i has
+    variance sigma^2 / s_i (appendix: variance reduction O(1/(nT)))."""
+    n, L, sigma, steps = 8, 20000, 1.0, 12
+    st = oracle.State(n, wl.binary_tree(n), L)
+    st.x, st.mu = np.zeros((n, L)), np.ones((n, L))
+    st.advance(steps, 0.0, sigma, 4, algo=oracle.ALGO_DME)
+    for i in range(n):
+        est = st.x[i] / st.dme_count[i]
+        assert abs(est.mean() - 1.0) < 5 * sigma / np.sqrt(st.dme_count[i] * L)
+        assert abs(est.var() * st.dme_count[i] / sigma ** 2 - 1.0) < 0.05
