@@ -353,60 +353,50 @@ def pinned_like(t):
 
 
 def run_e2e(args, w, run, dev, stream, world: int):
-    """relay_step with x, messages and counters living in pinned host memory:
-    every step copies them to the device, runs, and copies the results back."""
+    """The same metric through the host-state API: x, both message buffers and
+    the counters live in pinned host memory and every step streams them
+    through the GPU (HostRelayRun), copies inside the timed region."""
     import torch
 
-    import paper_2110_04175_gb300 as rs
+    from paper_2110_04175_gb300.host_stream import HostRelayRun
 
-    if len(run.trees) > 1:
+    if len(run.trees) > 1 or args.optimizer != "sgd" or args.algorithm != "relaysgd":
         return {"value": None, "unit": "steps/s",
-                "skipped": "host-buffer path measured on single-tree workloads"}
+                "skipped": "host-state path measured on single-tree SGD workloads"}
+    E = max(2 * (w.n - 1), 1)
 
     def pow2(b):  # the pinned allocator rounds every block up to a power of two
         return 1 << max(0, int(b - 1).bit_length())
-    need = pow2(run.x.numel() * 4) + 2 * pow2(run.msg[0].numel() * 4) + pow2(run.counts.numel() * 4)
+    cw = 1 << 22
+    nch = (w.d + cw - 1) // cw
+    need = pow2(nch * w.n * cw * 4) + 2 * pow2(nch * E * cw * 4)
     avail = host_mem_available()
     if need > 0.6 * avail:
         return {"value": None, "unit": "steps/s",
                 "skipped": f"pinned host state of {need / 1e9:.1f} GB exceeds 60% of the "
                            f"{avail / 1e9:.1f} GB available"}
-    hx = pinned_like(run.x)
-    hm_in = pinned_like(run.msg[0])
-    hm_out = pinned_like(run.msg[0])
-    hc = pinned_like(run.counts)
-    try:
-        hx.copy_(run.x)
-        hm_in.copy_(run.msg[run.cur])
-        hc.copy_(run.counts)
-        torch.cuda.synchronize(dev)
-        h2d = (hx.numel() + hm_in.numel() + hc.numel()) * 4
-        d2h = (hx.numel() + hm_out.numel() + hc.numel()) * 4
-        barrier(world)
-        start = torch.cuda.Event(enable_timing=True)
-        end = torch.cuda.Event(enable_timing=True)
-        start.record(stream)
-        for _ in range(args.e2e_steps):
-            run.x.copy_(hx, non_blocking=True)
-            run.msg[0].copy_(hm_in, non_blocking=True)
-            run.counts.copy_(hc, non_blocking=True)
-            rs.relay_step(run.h, run.x, run.msg[0], run.msg[1], run.counts, w.lr, w.seed, run.t,
-                          stream)
-            hx.copy_(run.x, non_blocking=True)
-            hm_out.copy_(run.msg[1], non_blocking=True)
-            hc.copy_(run.counts, non_blocking=True)
-            run.t += 1
-            hm_in, hm_out = hm_out, hm_in
-        end.record(stream)
-        torch.cuda.synchronize(dev)
-        ms = reduce_max(start.elapsed_time(end), world)
-    finally:
-        torch.cuda.synchronize(dev)
-        del hx, hm_in, hm_out, hc
+    # free the resident run's buffers first: the host run needs its own
+    del run.trees[:]
+    run.x = run.mu = None
+    torch.cuda.empty_cache()
+    host = HostRelayRun(w.n, w.d, w.edges, chunk=cw, device=dev, mode=w.mode,
+                        c0=shard_offset(int(os.environ.get("RANK", "0")), w.d))
+    host.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    host.step(w.lr, w.seed)  # warm-up
+    host.sync()
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        host.step(w.lr, w.seed)
+    host.sync()
+    ms = reduce_max((time.perf_counter() - t0) * 1e3, world)
+    h2d, d2h = host.bytes_per_step()
     return {"value": round(world * args.e2e_steps / (ms / 1e3), 4), "unit": "steps/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
-            "path": "relay_step with x, messages and counters in pinned host memory, "
-                    "copied in and out every step"}
+            "path": "HostRelayRun: state in pinned host memory, streamed through the GPU in "
+                    f"{host.nchunks} chunks of {cw} coordinates (copy-in / kernel / copy-out "
+                    "streams), copies inside the timed region",
+            "copy_gbs": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9, 1)}
 
 
 def traffic_per_launch(w, objective: str):
@@ -427,7 +417,7 @@ def main(argv=None):
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["native", "reference"], default="native")
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
-    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--e2e-steps", type=int, default=5)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--optimizer", choices=["sgd", "nesterov", "adam"], default="sgd",
                    help="local optimiser of the local step (appendix: momentum / Adam)")

@@ -1,0 +1,141 @@
+"""RelaySGD with the state in host memory, streamed through the GPU.
+
+For state larger than the GPU, or owned by the host, ``HostRelayRun`` keeps
+x, the two message buffers and the counters in pinned host memory, laid out
+in coordinate chunks (``[chunk][rows][cw]``, so each chunk of each array is
+one contiguous block).  A step:
+
+1. copies the counters in and runs the counter kernel once (Alg. 1 counters
+   are per edge, not per coordinate);
+2. streams the chunks through a ring of device buffers on three CUDA
+   streams -- host-to-device copies, the fused kernel (relay_step_models on
+   a handle whose coordinate offset is the chunk's absolute position), and
+   device-to-host copies -- so both copy directions and the kernels overlap;
+3. copies the counters out.
+
+Every coordinate of the method evolves independently and the noise is keyed
+by the absolute coordinate, so the result equals a run with the whole state
+resident on the device, bit for bit.  The centres are regenerated in the
+kernel (relay_set_objective_generated), so no device copy of mu is needed.
+All arithmetic runs in the library's kernels; this module only moves bytes
+and orders the streams.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from . import _native as nat
+
+
+class HostRelayRun:
+    """One tree, n workers, d coordinates, state in pinned host memory."""
+
+    def __init__(self, n: int, d: int, edges, chunk: int = 1 << 22, buffers: int = 3,
+                 device="cuda", mode: int = 1, c0: int = 0):
+        import torch
+        if chunk % 32 or chunk <= 0:
+            raise ValueError("chunk must be a positive multiple of 32")
+        self.n, self.d, self.c0, self.mode = n, d, c0, mode
+        self.device = torch.device(device)
+        self.cw = min(chunk, max(32, (d + 31) // 32 * 32))
+        self.nchunks = max(1, (d + self.cw - 1) // self.cw)
+        self.widths = [min(self.cw, d - k * self.cw) for k in range(self.nchunks)]
+        # one handle per distinct chunk width; the offset is set per launch
+        self.handles = {}
+        for wdt in sorted(set(self.widths)):
+            h = nat.relay_create(n, wdt, edges)
+            nat.relay_set_rebuild_mode(h, mode)
+            nat.relay_set_strides(h, self.cw, self.cw)
+            self.handles[wdt] = h
+        h0 = self.handles[self.widths[0]]
+        self.E = nat.relay_num_edges(h0)
+        E1 = max(self.E, 1)
+        pin = dict(dtype=torch.float32, pin_memory=True)
+        self.x_h = torch.empty(self.nchunks, n, self.cw, **pin)
+        self.msg_h = [torch.empty(self.nchunks, E1, self.cw, **pin) for _ in range(2)]
+        self.counts_h = torch.zeros(E1, dtype=torch.int32, pin_memory=True)
+        f32 = dict(dtype=torch.float32, device=self.device)
+        self.B = max(2, buffers)
+        self.xb = [torch.empty(n, self.cw, **f32) for _ in range(self.B)]
+        self.mib = [torch.empty(E1, self.cw, **f32) for _ in range(self.B)]
+        self.mob = [torch.empty(E1, self.cw, **f32) for _ in range(self.B)]
+        self.counts_d = torch.zeros(E1, dtype=torch.int32, device=self.device)
+        self.s_in = torch.cuda.Stream(self.device)
+        self.s_comp = torch.cuda.Stream(self.device)
+        self.s_out = torch.cuda.Stream(self.device)
+        self.in_done = [torch.cuda.Event() for _ in range(self.B)]
+        self.comp_done = [torch.cuda.Event() for _ in range(self.B)]
+        self.out_done = [torch.cuda.Event() for _ in range(self.B)]
+        self.counts_ready = torch.cuda.Event()
+        self.t = 0
+        self.cur = 0  # msg_h[cur] holds m^{t-1}
+
+    def _handle(self, k: int):
+        h = self.handles[self.widths[k]]
+        nat.relay_set_coord_offset(h, self.c0 + k * self.cw)
+        return h
+
+    def init(self, x0_std: float, seed: int, mix, mu_scale: float, mu_seed: int, sigma: float):
+        """x^0, zero messages and counters, written chunk by chunk on the device."""
+        import torch
+        mix = np.asarray(mix, dtype=np.float32)
+        for h in self.handles.values():
+            nat.relay_set_objective_generated(h, mix, mix.shape[1], mu_scale, mu_seed, sigma)
+        with torch.cuda.stream(self.s_comp):
+            for k in range(self.nchunks):
+                nat.relay_init(self._handle(k), self.xb[0], self.mib[0], None, self.counts_d,
+                               x0_std, seed, self.s_comp)
+                self.x_h[k].copy_(self.xb[0])
+                self.msg_h[0][k].copy_(self.mib[0])
+        self.counts_h.copy_(self.counts_d)
+        torch.cuda.synchronize(self.device)
+        self.t = 0
+        self.cur = 0
+
+    def step(self, lr: float, seed: int):
+        """Enqueues one RelaySGD step (asynchronous; call sync() to wait)."""
+        import torch
+        src, dst = self.msg_h[self.cur], self.msg_h[1 - self.cur]
+        with torch.cuda.stream(self.s_comp):
+            self.counts_d.copy_(self.counts_h, non_blocking=True)
+            nat.relay_step_counts(self.handles[self.widths[0]], self.counts_d, self.s_comp)
+            self.counts_ready.record(self.s_comp)
+        for k in range(self.nchunks):
+            b = k % self.B
+            with torch.cuda.stream(self.s_in):
+                self.s_in.wait_event(self.out_done[b])
+                self.xb[b].copy_(self.x_h[k], non_blocking=True)
+                self.mib[b].copy_(src[k], non_blocking=True)
+                self.in_done[b].record(self.s_in)
+            self.s_comp.wait_event(self.in_done[b])
+            nat.relay_step_models(self._handle(k), self.xb[b], self.mib[b], self.mob[b],
+                                  self.counts_d, lr, seed, self.t, self.s_comp)
+            self.comp_done[b].record(self.s_comp)
+            with torch.cuda.stream(self.s_out):
+                self.s_out.wait_event(self.comp_done[b])
+                self.x_h[k].copy_(self.xb[b], non_blocking=True)
+                dst[k].copy_(self.mob[b], non_blocking=True)
+                self.out_done[b].record(self.s_out)
+        with torch.cuda.stream(self.s_out):
+            self.s_out.wait_event(self.counts_ready)
+            self.counts_h.copy_(self.counts_d, non_blocking=True)
+        self.cur = 1 - self.cur
+        self.t += 1
+
+    def sync(self):
+        import torch
+        torch.cuda.synchronize(self.device)
+
+    def bytes_per_step(self):
+        """(host-to-device, device-to-host) bytes copied per step."""
+        h2d = (self.x_h.numel() + self.msg_h[0].numel() + self.counts_h.numel()) * 4
+        return h2d, h2d
+
+    def models(self):
+        """x as a host [n][d] array (a copy)."""
+        return self.x_h.permute(1, 0, 2).reshape(self.n, -1)[:, :self.d].clone()
+
+    def messages(self):
+        """m^{t-1} as a host [E][d] array (a copy)."""
+        m = self.msg_h[self.cur]
+        return m.permute(1, 0, 2).reshape(m.shape[1], -1)[:self.E, :self.d].clone()

@@ -1,0 +1,38 @@
+"""The host-state streaming mode equals the fully resident run, bit for bit."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2110_04175_gb300 as rs
+from paper_2110_04175_gb300 import workloads as wl
+from paper_2110_04175_gb300.host_stream import HostRelayRun
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+@pytest.mark.parametrize("shape,n,d,chunk,buffers", [
+    ("binary", 16, 1_000_003, 1 << 18, 3),   # 4 chunks, ragged last one
+    ("star", 12, 70_001, 1 << 14, 2),        # wide node, 5 chunks, 2 buffers
+    ("chain", 5, 1_000, 1 << 12, 3),         # a single chunk
+])
+def test_host_stream_equals_resident_run(shape, n, d, chunk, buffers):
+    edges = {"binary": wl.binary_tree(n), "star": wl.star(n), "chain": wl.chain(n)}[shape]
+    w = wl.Workload(shape, n, edges, d, wl.identity_mix(n), 1.0, 0.05, 0.05, 0.1, 7)
+    dev = rs.RelayRun(n, d, edges, device="cuda:0")
+    dev.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    host = HostRelayRun(n, d, edges, chunk=chunk, buffers=buffers, device="cuda:0")
+    host.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    for _ in range(w.steps):
+        dev.step(w.lr, w.seed)
+        host.step(w.lr, w.seed)
+    host.sync()
+    torch.cuda.synchronize()
+    assert torch.equal(host.models(), dev.x[:, :d].cpu())
+    assert torch.equal(host.messages(), dev.messages[:dev.E, :d].cpu())
+    assert torch.equal(host.counts_h[:dev.E], dev.counts[:dev.E].cpu())
