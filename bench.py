@@ -278,6 +278,8 @@ def run_native(args, w, rank: int, world: int):
     T = len(run.trees)
     for _ in range(args.warmup):
         one_step()
+    if args.graph:
+        return run_graphed(args, w, run, dev, stream, rank, world)
     events = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(T)]
               for _ in range(args.steps)]
     torch.cuda.synchronize(dev)
@@ -332,6 +334,41 @@ def run_native(args, w, rank: int, world: int):
             "config": workload_config(w, world, args), "roofline": roofline, "cpu_baseline": cpu,
             "e2e": e2e, "gpu_launches": 2 * T * args.steps, "clocks": clocks.summary(),
             "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1)}
+    print(json.dumps(line), flush=True)
+
+
+def run_graphed(args, w, run, dev, stream, rank: int, world: int):
+    """Timed region = one replay of a CUDA graph holding the K steps (for
+    launch-bound small problems); the graph is captured after the warm-up."""
+    import torch
+    torch.cuda.synchronize(dev)
+    g = run.capture(args.steps, w.lr, w.seed)
+    torch.cuda.synchronize(dev)
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    with ClockSampler(bus_id_of(dev.index or 0) if rank == 0 else None) as clocks:
+        start.record(stream)
+        g.replay()
+        end.record(stream)
+        torch.cuda.synchronize(dev)
+    total_ms = reduce_max(start.elapsed_time(end), world)
+    if rank != 0:
+        return
+    alg = w.bytes_per_step()
+    peak = measured_peaks().get("hbm_gbs") or FALLBACK_HBM_GBS
+    per_step = total_ms / args.steps
+    line = {"metric": METRIC, "value": round(world * args.steps / (total_ms / 1e3), 2),
+            "unit": "steps/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(per_step, 5), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": dict(workload_config(w, world, args), launch="one CUDA graph of K steps"),
+            "roofline": {"bound": "hbm", "achieved": round(alg / (per_step / 1e3) / 1e9, 1),
+                         "peak": peak, "unit": "GB/s",
+                         "frac": round(alg / (per_step / 1e3) / 1e9 / peak, 4), "traffic": None,
+                         "kernel": "whole step (graph replay)"},
+            "cpu_baseline": None, "e2e": None, "gpu_launches": 2 * len(run.trees) * args.steps,
+            "clocks": clocks.summary()}
     print(json.dumps(line), flush=True)
 
 
@@ -423,6 +460,8 @@ def main(argv=None):
                    help="local optimiser of the local step (appendix: momentum / Adam)")
     p.add_argument("--algorithm", choices=["relaysgd", "grad", "dme"], default="relaysgd",
                    help="Algorithm 1 (default), 6 (relayed updates) or 5 (mean estimation)")
+    p.add_argument("--graph", action="store_true",
+                   help="time one CUDA-graph replay of the K steps (small, launch-bound workloads)")
     p.add_argument("--lost-prob", type=float, default=0.0,
                    help="probability that each message is lost in transit, per step")
     p.add_argument("--objective", choices=["generated", "stored"], default="stored",

@@ -391,6 +391,21 @@ class RelayRun:
         self._mix = mix_t  # keep alive until the fills have run
         self.t = 0
 
+    def capture(self, steps: int, lr: float, seed: int):
+        """Records the next `steps` steps (t, t+1, ...) into one CUDA graph and
+        advances the run's bookkeeping as if they had run: replay the returned
+        graph exactly once to run them (the step counters are fixed in it).
+        For launch-bound small problems this replaces 2 launches per tree and
+        step by one graph launch."""
+        import torch
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream(self.device)
+        side.wait_stream(torch.cuda.current_stream(self.device))
+        with torch.cuda.graph(g, stream=side):
+            for _ in range(steps):
+                self.step(lr, seed, side)
+        return g
+
     def set_lost(self, lost, tree: int = 0):
         """Messages of the next steps lost in transit on tree `tree` (E flags or None)."""
         relay_set_lost_messages(self.trees[tree].h, lost)

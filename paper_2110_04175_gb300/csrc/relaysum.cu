@@ -146,7 +146,7 @@ __device__ __forceinline__ float4 fma4(float w, float4 z, float4 acc) {
 // Loads read once per step: read-only path, no L1 allocation.
 __device__ __forceinline__ float4 ld_stream(const float* p) {
     float4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
+    asm("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
                  : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
                  : "l"(p));
     return v;
@@ -155,8 +155,7 @@ __device__ __forceinline__ float4 ld_stream(const float* p) {
 // (program.h): keep them in L2 with evict-last priority until then.
 __device__ __forceinline__ float4 ld_keep(const float* p) {
     float4 v;
-    asm volatile(
-        "{\n\t.reg .b64 pol;\n\t"
+    asm("{\n\t.reg .b64 pol;\n\t"
         "createpolicy.fractional.L2::evict_last.b64 pol, 1.0;\n\t"
         "ld.global.nc.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], pol;\n\t}"
         : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
@@ -397,11 +396,22 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
                 cen[k * blockDim.x] = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k), 0u,
                                               1u, mu_key);
         }
+        // x (and a stored mu) of the next node in the walk are loaded one visit
+        // early, so their latency overlaps the current visit's arithmetic
+        float4 xn = *reinterpret_cast<const float4*>(a.x + prog.order[0] * a.ld_x + 4 * q);
+        float4 mn = (OBJ == relaysum::kMuStored) ? ld_stream(a.mu + prog.order[0] * a.ld_x + 4 * q)
+                                                  : make_float4(0.f, 0.f, 0.f, 0.f);
         for (int v = 0; v < n; ++v) {
             const int i = prog.order[v];
             const NodeRec r = prog.node[i];
-            const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
-            const float4 mv = centre<OBJ>(obj, mu_key, a, i, q, cen, static_cast<int>(blockDim.x));
+            const float4 xv = xn;
+            const float4 mv = (OBJ == relaysum::kMuStored)
+                                  ? mn : centre<OBJ>(obj, mu_key, a, i, q, cen, static_cast<int>(blockDim.x));
+            if (v + 1 < n) {  // the next node is never finalised before its own visit
+                const int inext = prog.order[v + 1];
+                xn = *reinterpret_cast<const float4*>(a.x + inext * a.ld_x + 4 * q);
+                if (OBJ == relaysum::kMuStored) mn = ld_stream(a.mu + inext * a.ld_x + 4 * q);
+            }
             const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i),
                                      a.step, 0u, a.key);
             // the relayed value: x^{t+1/2} = x + u (Alg. 1), the update u
@@ -548,11 +558,21 @@ int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream
             return RELAY_ECUDA;
         if (dev < kMaxDevices) smem_set[dev].store(true);
     }
+    // resident CTAs per SM, cached per device for the last shared-memory size
+    // (queried once, not per step: steps may be captured into CUDA graphs)
+    static std::atomic<int64_t> occ_cache[kMaxDevices];
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_models_kernel<OBJ, OPT>, threads, smem) !=
-            cudaSuccess ||
-        per_sm <= 0)
-        return RELAY_ECUDA;
+    const int64_t key = static_cast<int64_t>(smem) * 1024 + threads;
+    const int64_t cached = dev < kMaxDevices ? occ_cache[dev].load() : 0;
+    if (cached != 0 && (cached >> 8) == key) {
+        per_sm = static_cast<int>(cached & 0xFF);
+    } else {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_models_kernel<OBJ, OPT>, threads,
+                                                          smem) != cudaSuccess ||
+            per_sm <= 0)
+            return RELAY_ECUDA;
+        if (dev < kMaxDevices) occ_cache[dev].store((key << 8) | (per_sm & 0xFF));
+    }
     const int64_t want = (a.nquads + threads - 1) / threads;
     const int64_t cap = static_cast<int64_t>(sms) * per_sm;
     const int grid = static_cast<int>(want < cap ? want : cap);

@@ -13,6 +13,11 @@ one contiguous block).  A step:
    device-to-host copies -- so both copy directions and the kernels overlap;
 3. copies the counters out.
 
+Ordering: every reuse of a device buffer waits for the copy-out of the chunk
+that last used it; the next step's copy-in of a chunk waits (through the
+same buffer events, on in-order streams) for this step's copy-out of that
+chunk; and the counters' copy-in waits for the last step's copy-out.
+
 Every coordinate of the method evolves independently and the noise is keyed
 by the absolute coordinate, so the result equals a run with the whole state
 resident on the device, bit for bit.  The centres are regenerated in the
@@ -66,7 +71,8 @@ class HostRelayRun:
         self.in_done = [torch.cuda.Event() for _ in range(self.B)]
         self.comp_done = [torch.cuda.Event() for _ in range(self.B)]
         self.out_done = [torch.cuda.Event() for _ in range(self.B)]
-        self.counts_ready = torch.cuda.Event()
+        self.counts_ready = torch.cuda.Event()  # counter kernel of this step done
+        self.counts_saved = torch.cuda.Event()  # counters of the last step back on the host
         self.t = 0
         self.cur = 0  # msg_h[cur] holds m^{t-1}
 
@@ -97,6 +103,8 @@ class HostRelayRun:
         import torch
         src, dst = self.msg_h[self.cur], self.msg_h[1 - self.cur]
         with torch.cuda.stream(self.s_comp):
+            # the last step's counters must be back on the host before they go in again
+            self.s_comp.wait_event(self.counts_saved)
             self.counts_d.copy_(self.counts_h, non_blocking=True)
             nat.relay_step_counts(self.handles[self.widths[0]], self.counts_d, self.s_comp)
             self.counts_ready.record(self.s_comp)
@@ -119,6 +127,7 @@ class HostRelayRun:
         with torch.cuda.stream(self.s_out):
             self.s_out.wait_event(self.counts_ready)
             self.counts_h.copy_(self.counts_d, non_blocking=True)
+            self.counts_saved.record(self.s_out)
         self.cur = 1 - self.cur
         self.t += 1
 

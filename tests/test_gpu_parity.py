@@ -246,3 +246,20 @@ def test_binary16_resnet20_every_coordinate_mode0():
     assert parity_error(gx, st.x) <= RTOL
     assert parity_error(gm, st.msg) <= RTOL
     assert np.array_equal(run.counts.cpu().numpy(), st.counts)
+
+
+def test_captured_graph_equals_eager_steps():
+    """A CUDA graph of K captured steps, replayed once, gives the eager run."""
+    w = wl.chain8_d4096()
+    eager = gpu_run(w, 30)
+    run = rs.RelayRun(w.n, w.d, w.edges, device="cuda:0")
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    for _ in range(10):
+        run.step(w.lr, w.seed)
+    g = run.capture(20, w.lr, w.seed)
+    g.replay()
+    torch.cuda.synchronize()
+    assert run.t == 30
+    assert torch.equal(run.x[:, :w.d], eager.x[:, :w.d])
+    assert torch.equal(run.messages[:, :w.d], eager.messages[:, :w.d])
+    assert torch.equal(run.counts, eager.counts)
