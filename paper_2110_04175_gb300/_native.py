@@ -391,6 +391,32 @@ class RelayRun:
         self._mix = mix_t  # keep alive until the fills have run
         self.t = 0
 
+    def state_dict(self) -> dict:
+        """The run's full state as host tensors: models, both message buffers,
+        counters, optimiser state, mean-estimation counts, step and buffer
+        parity.  With the seeds, it resumes the run bit for bit."""
+        sd = {"t": self.t, "x": self.x.cpu(), "state": [s.cpu() for s in self.state],
+              "trees": [{"cur": tr.cur, "msg": [m.cpu() for m in tr.msg],
+                         "counts": tr.counts.cpu(),
+                         "dme_count": None if tr.dme_count is None else tr.dme_count.cpu()}
+                        for tr in self.trees]}
+        return sd
+
+    def load_state_dict(self, sd: dict):
+        """Restores a state_dict() into this run (same n, d, trees and options;
+        init() must have bound the objective first)."""
+        self.t = int(sd["t"])
+        self.x.copy_(sd["x"])
+        for dst, src in zip(self.state, sd["state"]):
+            dst.copy_(src)
+        for tr, st in zip(self.trees, sd["trees"]):
+            tr.cur = int(st["cur"])
+            for dst, src in zip(tr.msg, st["msg"]):
+                dst.copy_(src)
+            tr.counts.copy_(st["counts"])
+            if tr.dme_count is not None:
+                tr.dme_count.copy_(st["dme_count"])
+
     def capture(self, steps: int, lr: float, seed: int):
         """Records the next `steps` steps (t, t+1, ...) into one CUDA graph and
         advances the run's bookkeeping as if they had run: replay the returned

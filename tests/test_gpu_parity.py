@@ -263,3 +263,33 @@ def test_captured_graph_equals_eager_steps():
     assert torch.equal(run.x[:, :w.d], eager.x[:, :w.d])
     assert torch.equal(run.messages[:, :w.d], eager.messages[:, :w.d])
     assert torch.equal(run.counts, eager.counts)
+
+
+@pytest.mark.parametrize("optimizer,algorithm", [(None, "relaysgd"), (("adam", 0.9, 0.99, 1e-8), "relaysgd"),
+                                                 (None, "dme")])
+def test_checkpoint_resume_is_bit_exact(optimizer, algorithm):
+    """Save the full state after k steps, restore it into a fresh run, take k
+    more steps: identical to 2k uninterrupted steps."""
+    w = wl.sweep64("star")
+    w.d = 20_000
+    kw = dict(device="cuda:0", optimizer=optimizer, algorithm=algorithm)
+    a = rs.RelayRun(w.n, w.d, w.edges, **kw)
+    a.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    for _ in range(12):
+        a.step(w.lr, w.seed)
+    b = rs.RelayRun(w.n, w.d, w.edges, **kw)
+    b.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    for _ in range(6):
+        b.step(w.lr, w.seed)
+    sd = b.state_dict()
+    c = rs.RelayRun(w.n, w.d, w.edges, **kw)
+    c.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    c.load_state_dict(sd)
+    for _ in range(6):
+        c.step(w.lr, w.seed)
+    torch.cuda.synchronize()
+    assert torch.equal(a.x[:, :w.d], c.x[:, :w.d])
+    assert torch.equal(a.messages[:, :w.d], c.messages[:, :w.d])
+    assert torch.equal(a.counts, c.counts)
+    if algorithm == "dme":
+        assert torch.equal(a.trees[0].dme_count, c.trees[0].dme_count)
