@@ -438,13 +438,18 @@ def run_e2e(args, w, run, dev, stream, world: int):
 
 def traffic_per_launch(w, objective: str):
     """DRAM bytes per launch of the fused kernel from the committed ncu
-    summary for this workload and objective source, if one exists."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    summary for this workload and objective source (profiles/traffic.txt),
+    or None when no capture of the current kernel exists for it."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
     try:
         with open(path) as f:
-            return json.load(f).get(f"{w.name}/{objective}")
-    except (OSError, ValueError):
-        return None
+            for line in f:
+                parts = line.split()
+                if len(parts) == 2 and not line.startswith("#") and parts[0] == f"{w.name}/{objective}":
+                    return int(parts[1])
+    except OSError:
+        pass
+    return None
 
 
 def main(argv=None):

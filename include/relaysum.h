@@ -201,6 +201,18 @@ int relay_nbar(const relay_handle *h, const int32_t *counts_host, int32_t *nbar_
 int relay_program(const relay_handle *h, int32_t *nslots, int32_t *order, int32_t *node_rec,
                   int32_t *pos_rec);
 
+/* Convergence metrics of the current models x (device [n][ld_x]): out[0] =
+ * the consensus distance 1/(n d) sum_i ||x_i - xbar||^2, out[1] = the
+ * distance of the average model to the optimum ||xbar - mubar||^2 / d, where
+ * xbar, mubar are the worker averages (the quantities of Section 4's
+ * analysis; mubar is the optimum of f = 1/n sum_i f_i).  out: device double
+ * [2]; workspace: device double [relay_metrics_workspace(h)], caller-owned
+ * scratch for per-block partial sums, overwritten by every call.  Reduced in
+ * double in a fixed order: deterministic.  Needs a bound objective. */
+int64_t relay_metrics_workspace(const relay_handle *h);
+int relay_metrics(relay_handle *h, const float *x, double *workspace, double *out,
+                  relay_stream_t stream);
+
 /* Static description of a status code. */
 const char *relay_error_string(int status);
 

@@ -64,6 +64,8 @@ def _load():
             "relay_step": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, vp]),
             "relay_nbar": (ctypes.c_int, [vp, vp, vp]),
             "relay_program": (ctypes.c_int, [vp, vp, vp, vp, vp]),
+            "relay_metrics_workspace": (i64, [vp]),
+            "relay_metrics": (ctypes.c_int, [vp, vp, vp, vp, vp]),
             "relay_error_string": (ctypes.c_char_p, [ctypes.c_int]),
         }
         for name, (res, args) in sig.items():
@@ -240,6 +242,16 @@ def relay_step(h, x, msg_in, msg_out, counts, lr: float, seed: int, step: int, s
                               float(lr), int(seed), int(step), _stream(stream)), "relay_step")
 
 
+def relay_metrics_workspace(h) -> int:
+    return int(_load().relay_metrics_workspace(_h(h)))
+
+
+def relay_metrics(h, x, workspace, out, stream=None):
+    """out (device float64 [2]) = (consensus distance, distance to the optimum)."""
+    _check(_load().relay_metrics(_h(h), _ptr(x), _ptr(workspace), _ptr(out), _stream(stream)),
+           "relay_metrics")
+
+
 def relay_nbar(h, counts_host) -> np.ndarray:
     c = np.ascontiguousarray(np.asarray(counts_host, dtype=np.int32))
     n = h.n if isinstance(h, RelayHandle) else None
@@ -390,6 +402,18 @@ class RelayRun:
             tr.cur = 0
         self._mix = mix_t  # keep alive until the fills have run
         self.t = 0
+
+    def metrics(self):
+        """(consensus distance, distance of the average model to the optimum)
+        of the current models, as a device float64 tensor [trees][2]."""
+        import torch
+        out = torch.zeros(len(self.trees), 2, dtype=torch.float64, device=self.device)
+        for k, tr in enumerate(self.trees):
+            if tr.d == 0:
+                continue
+            ws = torch.empty(relay_metrics_workspace(tr.h), dtype=torch.float64, device=self.device)
+            relay_metrics(tr.h, self._x(tr), ws, out[k])
+        return out
 
     def state_dict(self) -> dict:
         """The run's full state as host tensors: models, both message buffers,

@@ -19,6 +19,7 @@
 //   relay_fill_mu_kernel  mu_i = scale * sum_k mix[i][k] N_k.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <atomic>
 #include <cmath>
 #include <cstdint>
@@ -501,6 +502,83 @@ __global__ void relay_fill_mu_kernel(float* mu, const float* mix, int n, int K, 
     }
 }
 
+// ------------------------------------------------------------------ metrics
+
+// Consensus distance and distance to the optimum (the quantities of the
+// paper's analysis, Section 4): per coordinate c, with xbar = mean_i x_i and
+// mubar = mean_i mu_i,
+//   xi   += sum_i (x_i - xbar)^2        dist += (xbar - mubar)^2
+// accumulated in double.  Pass 1: each block reduces its share of the
+// coordinates (grid-stride, fixed order) into partials[2 blockIdx];
+// pass 2 sums the partials in a fixed order, so the result is deterministic.
+constexpr int kMetricsThreads = 256;
+constexpr int kMetricsMaxBlocks = 1024;
+
+__device__ __forceinline__ double block_sum(double v, double* red) {
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    __syncthreads();
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    double s = 0.0;
+    if (threadIdx.x == 0)
+        for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) s += red[w];
+    return s;  // valid in thread 0
+}
+
+template <int OBJ>
+__global__ void __launch_bounds__(kMetricsThreads)
+relay_metrics_kernel(const __grid_constant__ Objective obj, const __grid_constant__ PhiloxKey mu_key,
+                     const __grid_constant__ ModelArgs a, int n, int64_t d, double* partials) {
+    __shared__ double red[kMetricsThreads / 32];
+    double xi = 0.0, dist = 0.0;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < a.nquads; q += stride) {
+        double xs[4] = {0, 0, 0, 0}, ms[4] = {0, 0, 0, 0};
+        for (int i = 0; i < n; ++i) {
+            const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
+            const float4 mv = centre<OBJ>(obj, mu_key, a, i, q, nullptr, 0);
+            xs[0] += xv.x; xs[1] += xv.y; xs[2] += xv.z; xs[3] += xv.w;
+            ms[0] += mv.x; ms[1] += mv.y; ms[2] += mv.z; ms[3] += mv.w;
+        }
+        double xb[4], ss[4] = {0, 0, 0, 0};
+        for (int k = 0; k < 4; ++k) xb[k] = xs[k] / n;
+        for (int i = 0; i < n; ++i) {
+            const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
+            const double dv[4] = {xv.x - xb[0], xv.y - xb[1], xv.z - xb[2], xv.w - xb[3]};
+            for (int k = 0; k < 4; ++k) ss[k] += dv[k] * dv[k];
+        }
+        for (int k = 0; k < 4; ++k)
+            if (4 * q + k < d) {
+                xi += ss[k];
+                const double e = xb[k] - ms[k] / n;
+                dist += e * e;
+            }
+    }
+    const double bxi = block_sum(xi, red);
+    const double bdist = block_sum(dist, red);
+    if (threadIdx.x == 0) {
+        partials[2 * blockIdx.x] = bxi;
+        partials[2 * blockIdx.x + 1] = bdist;
+    }
+}
+
+__global__ void relay_metrics_finish_kernel(const double* partials, int blocks, double scale_xi,
+                                            double scale_dist, double* out) {
+    __shared__ double red[kMetricsThreads / 32];
+    double xi = 0.0, dist = 0.0;
+    for (int b = threadIdx.x; b < blocks; b += blockDim.x) {
+        xi += partials[2 * b];
+        dist += partials[2 * b + 1];
+    }
+    const double sxi = block_sum(xi, red);
+    const double sdist = block_sum(dist, red);
+    if (threadIdx.x == 0) {
+        out[0] = sxi * scale_xi;
+        out[1] = sdist * scale_dist;
+    }
+}
+
 // ------------------------------------------------------------- host helpers
 
 constexpr int kMaxDevices = 64;
@@ -912,6 +990,41 @@ int relay_program(const relay_handle* h, int32_t* nslots, int32_t* order, int32_
             pos_rec[3 * e + 2] = p.pos_slot[e];
         }
     return RELAY_OK;
+}
+
+int64_t relay_metrics_workspace(const relay_handle* h) {
+    if (!h) return RELAY_EINVAL;
+    const int64_t blocks = (h->nquads + kMetricsThreads - 1) / kMetricsThreads;
+    return 2 * std::max<int64_t>(1, std::min<int64_t>(blocks, kMetricsMaxBlocks));
+}
+
+int relay_metrics(relay_handle* h, const float* x, double* workspace, double* out, relay_stream_t stream) {
+    if (!h || !h->has_objective || !out || !workspace) return RELAY_EINVAL;
+    if (h->d > 0 && (!x || !aligned16(x))) return RELAY_EINVAL;
+    const int blocks = static_cast<int>(relay_metrics_workspace(h) / 2);
+    ModelArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.x = const_cast<float*>(x);
+    a.mu = h->mu;
+    a.ld_x = h->ld_x;
+    a.nquads = h->nquads;
+    a.q0 = static_cast<uint32_t>(h->c0 / 4);
+    const PhiloxKey mu_key = philox_key(static_cast<uint64_t>(h->obj.k0) | (static_cast<uint64_t>(h->obj.k1) << 32));
+    const int n = h->prog.n;
+    switch (h->obj.source) {
+        case relaysum::kMuStored:
+            relay_metrics_kernel<relaysum::kMuStored><<<blocks, kMetricsThreads, 0, stream>>>(
+                h->obj, mu_key, a, n, h->d, workspace);
+            break;
+        default:  // cached centres are regenerated per row here
+            relay_metrics_kernel<relaysum::kMuPerRow><<<blocks, kMetricsThreads, 0, stream>>>(
+                h->obj, mu_key, a, n, h->d, workspace);
+            break;
+    }
+    const double denom = h->d > 0 ? static_cast<double>(h->d) : 1.0;
+    relay_metrics_finish_kernel<<<1, kMetricsThreads, 0, stream>>>(workspace, blocks, 1.0 / (n * denom),
+                                                                   1.0 / denom, out);
+    return launch_status();
 }
 
 const char* relay_error_string(int status) {
