@@ -213,6 +213,24 @@ int64_t relay_metrics_workspace(const relay_handle *h);
 int relay_metrics(relay_handle *h, const float *x, double *workspace, double *out,
                   relay_stream_t stream);
 
+/* relay_metrics without a workspace argument, for callers that cannot
+ * allocate device memory: code that runs while a CUDA graph is being
+ * captured in global mode (where cudaMalloc is refused), or a host that
+ * hands all device memory to its own pool and gives a plug-in none.  The
+ * per-block partial sums go to a scratch array of 2 x 1024 doubles (16 KB)
+ * built into the library, which every GPU that loads the library holds until
+ * the process exits; nothing is allocated, and each call overwrites every
+ * partial it reads, so no state carries over between calls.  The first call
+ * on a device looks the array's address up (cudaGetSymbolAddress) with that
+ * device current, so make it before any stream capture.  The caller still
+ * passes x and out (device double [2]).  All calls share the one array:
+ * calls whose work overlaps on the GPU (different streams, or different
+ * host threads) race, so order them.  RELAY_EUNSUPPORTED if the reduction
+ * would need more than 1024 partial blocks (it never does: the block count
+ * is capped there).  The paper has no counterpart: this is a library
+ * convenience. */
+int relay_metrics_static(relay_handle *h, const float *x, double *out, relay_stream_t stream);
+
 /* Static description of a status code. */
 const char *relay_error_string(int status);
 

@@ -19,7 +19,7 @@ from ._native import (RELAY_EINVAL, RELAY_ECUDA, RELAY_ENOMEM, RELAY_ENOTTREE, R
                       RelayError, RelayHandle, RelayRun, library_path,
                       relay_create, relay_destroy, relay_edges, relay_error_string,
                       relay_fill_objective, relay_init, relay_ld, relay_metrics,
-                      relay_metrics_workspace, relay_nbar, relay_num_edges,
+                      relay_metrics_static, relay_metrics_workspace, relay_nbar, relay_num_edges,
                       relay_program, relay_set_coord_offset, relay_set_objective,
                       relay_set_algorithm, relay_set_local_optimizer, relay_set_lost_messages,
                       relay_set_objective_generated, relay_set_rebuild_mode, relay_set_strides,
@@ -36,5 +36,6 @@ __all__ = [
     "relay_set_objective_generated", "relay_fill_objective", "relay_init", "relay_step_counts",
     "relay_step_models", "relay_step",
     "relay_nbar", "relay_program", "relay_metrics", "relay_metrics_workspace",
+    "relay_metrics_static",
     "relay_error_string",
 ]

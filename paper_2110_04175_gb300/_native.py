@@ -66,6 +66,7 @@ def _load():
             "relay_program": (ctypes.c_int, [vp, vp, vp, vp, vp]),
             "relay_metrics_workspace": (i64, [vp]),
             "relay_metrics": (ctypes.c_int, [vp, vp, vp, vp, vp]),
+            "relay_metrics_static": (ctypes.c_int, [vp, vp, vp, vp]),
             "relay_error_string": (ctypes.c_char_p, [ctypes.c_int]),
         }
         for name, (res, args) in sig.items():
@@ -250,6 +251,12 @@ def relay_metrics(h, x, workspace, out, stream=None):
     """out (device float64 [2]) = (consensus distance, distance to the optimum)."""
     _check(_load().relay_metrics(_h(h), _ptr(x), _ptr(workspace), _ptr(out), _stream(stream)),
            "relay_metrics")
+
+
+def relay_metrics_static(h, x, out, stream=None):
+    """relay_metrics with the library's built-in scratch: allocates nothing."""
+    _check(_load().relay_metrics_static(_h(h), _ptr(x), _ptr(out), _stream(stream)),
+           "relay_metrics_static")
 
 
 def relay_nbar(h, counts_host) -> np.ndarray:

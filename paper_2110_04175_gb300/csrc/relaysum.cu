@@ -1027,6 +1027,40 @@ int relay_metrics(relay_handle* h, const float* x, double* workspace, double* ou
     return launch_status();
 }
 
+// ------------------------------------------- allocation-free metrics variant
+
+// Scratch for relay_metrics_static: the per-block partial sums of the metrics
+// reduction, in a file-scope device array instead of a caller workspace.
+// Every GPU that loads the library holds it (16 KB) until the process exits.
+constexpr int kStaticMetricsDoubles = 2 * kMetricsMaxBlocks;
+static __device__ __align__(256) double g_metrics_scratch[kStaticMetricsDoubles];
+
+namespace {
+// The array's device address, looked up once per device with that device
+// current.  (In host code the array's name is only a host-side stand-in.)
+std::atomic<double*> g_metrics_scratch_addr[kMaxDevices];
+
+double* metrics_scratch_address(int dev) {
+    double* p = dev < kMaxDevices ? g_metrics_scratch_addr[dev].load() : nullptr;
+    if (p) return p;
+    if (cudaGetSymbolAddress(reinterpret_cast<void**>(&p), g_metrics_scratch) != cudaSuccess || !p)
+        return nullptr;
+    if (dev < kMaxDevices) g_metrics_scratch_addr[dev].store(p);
+    return p;
+}
+}  // namespace
+
+int relay_metrics_static(relay_handle* h, const float* x, double* out, relay_stream_t stream) {
+    if (!h) return RELAY_EINVAL;
+    if (relay_metrics_workspace(h) > kStaticMetricsDoubles) return RELAY_EUNSUPPORTED;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return RELAY_ECUDA;
+    double* scratch = metrics_scratch_address(dev);
+    if (!scratch) return RELAY_ECUDA;
+    // pass 1 overwrites every partial that pass 2 reads: nothing to clear
+    return relay_metrics(h, x, scratch, out, stream);
+}
+
 const char* relay_error_string(int status) {
     switch (status) {
         case RELAY_OK: return "ok";
