@@ -417,7 +417,8 @@ def run_e2e(args, w, run, dev, stream, world: int):
     run.x = run.mu = None
     torch.cuda.empty_cache()
     host = HostRelayRun(w.n, w.d, w.edges, chunk=cw, device=dev, mode=w.mode,
-                        c0=shard_offset(int(os.environ.get("RANK", "0")), w.d))
+                        c0=shard_offset(int(os.environ.get("RANK", "0")), w.d),
+                        copy_streams=args.copy_streams)
     host.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
     host.step(w.lr, w.seed)  # warm-up
     host.sync()
@@ -431,8 +432,8 @@ def run_e2e(args, w, run, dev, stream, world: int):
     return {"value": round(world * args.e2e_steps / (ms / 1e3), 4), "unit": "steps/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
             "path": "HostRelayRun: state in pinned host memory, streamed through the GPU in "
-                    f"{host.nchunks} chunks of {cw} coordinates (copy-in / kernel / copy-out "
-                    "streams), copies inside the timed region",
+                    f"{host.nchunks} chunks of {cw} coordinates ({args.copy_streams} copy-in / "
+                    f"kernel / {args.copy_streams} copy-out streams), copies inside the timed region",
             "copy_gbs": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9, 1)}
 
 
@@ -460,6 +461,8 @@ def main(argv=None):
     p.add_argument("--impl", choices=["native", "reference"], default="native")
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     p.add_argument("--e2e-steps", type=int, default=5)
+    p.add_argument("--copy-streams", type=int, default=2,
+                   help="copy streams per direction of the host-state path")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--optimizer", choices=["sgd", "nesterov", "adam"], default="sgd",
                    help="local optimiser of the local step (appendix: momentum / Adam)")

@@ -14,9 +14,10 @@ one contiguous block).  A step:
 3. copies the counters out.
 
 Ordering: every reuse of a device buffer waits for the copy-out of the chunk
-that last used it; the next step's copy-in of a chunk waits (through the
-same buffer events, on in-order streams) for this step's copy-out of that
-chunk; and the counters' copy-in waits for the last step's copy-out.
+that last used it; a chunk's copy-in waits for the previous step's copy-out
+of the same chunk (an event per chunk, as copies alternate between several
+streams per direction); and the counters' copy-in waits for the last step's
+copy-out.
 
 Every coordinate of the method evolves independently and the noise is keyed
 by the absolute coordinate, so the result equals a run with the whole state
@@ -36,7 +37,7 @@ class HostRelayRun:
     """One tree, n workers, d coordinates, state in pinned host memory."""
 
     def __init__(self, n: int, d: int, edges, chunk: int = 1 << 22, buffers: int = 3,
-                 device="cuda", mode: int = 1, c0: int = 0):
+                 device="cuda", mode: int = 1, c0: int = 0, copy_streams: int = 2):
         import torch
         if chunk % 32 or chunk <= 0:
             raise ValueError("chunk must be a positive multiple of 32")
@@ -60,17 +61,21 @@ class HostRelayRun:
         self.msg_h = [torch.empty(self.nchunks, E1, self.cw, **pin) for _ in range(2)]
         self.counts_h = torch.zeros(E1, dtype=torch.int32, pin_memory=True)
         f32 = dict(dtype=torch.float32, device=self.device)
-        self.B = max(2, buffers)
+        self.B = max(2, buffers, copy_streams)
         self.xb = [torch.empty(n, self.cw, **f32) for _ in range(self.B)]
         self.mib = [torch.empty(E1, self.cw, **f32) for _ in range(self.B)]
         self.mob = [torch.empty(E1, self.cw, **f32) for _ in range(self.B)]
         self.counts_d = torch.zeros(E1, dtype=torch.int32, device=self.device)
-        self.s_in = torch.cuda.Stream(self.device)
+        # copies in each direction alternate between `copy_streams` streams so
+        # that several copy engines can work at once
+        self.s_ins = [torch.cuda.Stream(self.device) for _ in range(copy_streams)]
+        self.s_outs = [torch.cuda.Stream(self.device) for _ in range(copy_streams)]
+        self.s_in, self.s_out = self.s_ins[0], self.s_outs[0]
         self.s_comp = torch.cuda.Stream(self.device)
-        self.s_out = torch.cuda.Stream(self.device)
         self.in_done = [torch.cuda.Event() for _ in range(self.B)]
         self.comp_done = [torch.cuda.Event() for _ in range(self.B)]
         self.out_done = [torch.cuda.Event() for _ in range(self.B)]
+        self.out_done_k = [torch.cuda.Event() for _ in range(self.nchunks)]  # chunk k written back
         self.counts_ready = torch.cuda.Event()  # counter kernel of this step done
         self.counts_saved = torch.cuda.Event()  # counters of the last step back on the host
         self.t = 0
@@ -110,20 +115,26 @@ class HostRelayRun:
             self.counts_ready.record(self.s_comp)
         for k in range(self.nchunks):
             b = k % self.B
-            with torch.cuda.stream(self.s_in):
-                self.s_in.wait_event(self.out_done[b])
+            s_in = self.s_ins[k % len(self.s_ins)]
+            s_out = self.s_outs[k % len(self.s_outs)]
+            with torch.cuda.stream(s_in):
+                # the buffer's last chunk is out, and (through the same event on
+                # in-order streams) so is this chunk's output of the last step
+                s_in.wait_event(self.out_done[b])
+                s_in.wait_event(self.out_done_k[k])
                 self.xb[b].copy_(self.x_h[k], non_blocking=True)
                 self.mib[b].copy_(src[k], non_blocking=True)
-                self.in_done[b].record(self.s_in)
+                self.in_done[b].record(s_in)
             self.s_comp.wait_event(self.in_done[b])
             nat.relay_step_models(self._handle(k), self.xb[b], self.mib[b], self.mob[b],
                                   self.counts_d, lr, seed, self.t, self.s_comp)
             self.comp_done[b].record(self.s_comp)
-            with torch.cuda.stream(self.s_out):
-                self.s_out.wait_event(self.comp_done[b])
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(self.comp_done[b])
                 self.x_h[k].copy_(self.xb[b], non_blocking=True)
                 dst[k].copy_(self.mob[b], non_blocking=True)
-                self.out_done[b].record(self.s_out)
+                self.out_done[b].record(s_out)
+                self.out_done_k[k].record(s_out)
         with torch.cuda.stream(self.s_out):
             self.s_out.wait_event(self.counts_ready)
             self.counts_h.copy_(self.counts_d, non_blocking=True)
