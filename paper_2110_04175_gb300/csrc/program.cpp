@@ -6,10 +6,10 @@
 // reverse), sorts every worker's neighbours by id, and then lays out the
 // depth-first walk described in program.h so that it needs as few
 // shared-memory slots per thread as possible:
-//   - children are visited in decreasing order of the slots their subtrees
-//     need (the classic register-allocation order for trees), so the
-//     messages still waiting for later siblings are few while a large
-//     subtree is walked;
+//   - children are ordered so that the costliest subtree comes last (a
+//     parent's slots die at its last child's visit, so that subtree runs
+//     almost free) and the others in decreasing need (fewer sibling messages
+//     wait while a large subtree is walked);
 //   - every worker is tried as the root and the cheapest walk is kept.
 #include "program.h"
 
@@ -113,23 +113,53 @@ Walk make_walk(const Tree& t, int root) {
                 bfs.push_back(j);
             }
     }
-    std::vector<int> need(n, 0);
+    // need[i]: peak slots live during i's visit and its subtree, counting i's
+    // incoming slot.  A parent's accumulator (and a wide parent's total) dies
+    // at the end of its LAST child's visit, and no sibling message is pending
+    // then, so the last child's subtree runs almost free: the best order puts
+    // the costliest child last and the others in decreasing need.  Every
+    // child is tried as the last one.
+    std::vector<int> need(n, 0), vpeak(n, 0);
     for (int q = n - 1; q >= 0; --q) {
         const int i = bfs[q];
         auto& ch = w.children[i];
-        std::stable_sort(ch.begin(), ch.end(), [&](int a, int b) { return need[a] > need[b]; });
         const int m = static_cast<int>(ch.size());
         const int D = static_cast<int>(t.nbr[i].size());
-        // slots held by i while its children's subtrees are walked:
-        // narrow: accumulator + one pending message per later child;
-        // wide: accumulator + total (children read the total, no pending messages)
         const bool wide = D > kRegDeg;
-        int peak = (w.parent[i] >= 0) ? 1 : 0;
-        const int own = (m > 0) ? (wide ? 2 : 1) : 0;
-        peak = std::max(peak, own + (wide ? 0 : m));
-        for (int k = 0; k < m; ++k)
-            peak = std::max(peak, own + (wide ? 0 : (m - 1 - k)) + need[ch[k]] - (wide ? 1 : 0));
-        need[i] = std::max(peak, 1);
+        const int has_parent = w.parent[i] >= 0 ? 1 : 0;
+        const int own = (m > 0) ? (wide ? 2 : 1) : 0;             // accumulator (+ total)
+        vpeak[i] = std::max(has_parent, own + (wide ? 0 : m));     // slots at i's own visit
+        std::stable_sort(ch.begin(), ch.end(), [&](int a, int b) { return need[a] > need[b]; });
+        auto peak_of = [&](const std::vector<int>& order) {
+            int peak = vpeak[i];
+            for (int k = 0; k < m; ++k) {
+                const int c = order[k];
+                const int pending = wide ? 0 : (m - 1 - k);        // messages to later children
+                const int shared = wide ? 1 : 0;                   // a wide parent's total is c's input
+                if (k < m - 1) {
+                    peak = std::max(peak, own + pending + need[c] - shared);
+                } else {  // last child: i's slots live only through c's own visit
+                    peak = std::max(peak, own + vpeak[c] - shared);
+                    peak = std::max(peak, need[c]);
+                }
+            }
+            return peak;
+        };
+        int best = peak_of(ch);
+        std::vector<int> best_order = ch;
+        for (int last = 0; last < m; ++last) {
+            std::vector<int> order;
+            for (int k = 0; k < m; ++k)
+                if (k != last) order.push_back(ch[k]);
+            order.push_back(ch[last]);
+            const int p = peak_of(order);
+            if (p < best) {
+                best = p;
+                best_order = order;
+            }
+        }
+        ch = best_order;
+        need[i] = std::max(best, 1);
     }
     // pre-order
     std::vector<int> stack{root};
