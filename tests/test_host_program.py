@@ -273,3 +273,12 @@ def test_step_rejects_bad_arguments_before_any_launch():
     assert lib.relay_step(h.raw, fake, big, 2 * big, fake, float("nan"), 0, 0, None) == rs.RELAY_EINVAL
     assert lib.relay_step(h.raw, fake, fake + 256, 2 * big, fake, 0.1, 0, 0, None) == rs.RELAY_EINVAL
     assert lib.relay_step(h.raw, fake, big, 2 * big, fake, 0.1, 0, 1 << 32, None) == rs.RELAY_EINVAL
+
+
+def test_binding_fails_loudly_without_the_library(monkeypatch, tmp_path):
+    """No CPU fallback: with the shared library absent, the first call raises."""
+    from paper_2110_04175_gb300 import _native
+    monkeypatch.setattr(_native, "_lib", None)
+    monkeypatch.setattr(rs_build, "LIB", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        rs.relay_create(3, 8, wl.chain(3))
