@@ -287,7 +287,10 @@ __device__ __forceinline__ void visit_small(const Program& prog, const NodeRec& 
 
 // Degree D > kRegDeg: one streaming pass forms T = xh + sum of all incoming
 // messages; the message to the parent is T minus the parent's incoming
-// message, and T stays in a slot for the children (see program.h).
+// message, and T stays in a slot for the children (see program.h).  The
+// pass runs over descending positions while the children are visited in
+// ascending order, so the first children re-read the most recently read
+// (L2-resident) rows.
 __device__ __noinline__ void visit_wide(const Program& prog, const NodeRec& r, const ModelArgs& a,
                                         int64_t q, float4 xh, const Slots& sl,
                                         const float* s_scale) {
@@ -295,7 +298,7 @@ __device__ __noinline__ void visit_wide(const Program& prog, const NodeRec& r, c
     const int base = r.pos_base;
     float4 total = xh;
     float4 from_parent = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s = 0; s < D; ++s) {
+    for (int s = D - 1; s >= 0; --s) {
         const float4 m = ld_keep(a.msg_in + prog.pos_in[base + s] * a.ld_m + 4 * q);
         total = add4(total, m);
         if (s == r.parent_pos) from_parent = m;
