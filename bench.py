@@ -60,6 +60,11 @@ def reduce_max(value: float, world: int) -> float:
     return float(t.item())
 
 
+def reduce_min(value: float, world: int) -> float:
+    """Min over ranks (used for decisions every rank must take alike)."""
+    return -reduce_max(-value, world)
+
+
 def barrier(world: int):
     if world > 1:
         import torch.distributed as dist
@@ -410,7 +415,8 @@ def run_e2e(args, w, run, dev, stream, world: int):
     # every rank on this node pins its own state: split the host's memory
     local_world = max(1, int(os.environ.get("LOCAL_WORLD_SIZE", str(world))))
     avail = host_mem_available()
-    if need > 0.6 * avail / local_world:
+    # all ranks take the same decision (they enter a barrier below)
+    if reduce_min(1.0 if need <= 0.6 * avail / local_world else 0.0, world) < 0.5:
         return {"value": None, "unit": "steps/s",
                 "skipped": f"pinned host state of {need / 1e9:.1f} GB per rank exceeds 60% of the "
                            f"{avail / 1e9:.1f} GB available split over {local_world} rank(s)"}

@@ -31,9 +31,10 @@ def _worker(rank, world, port, result_dir):
         from oracle import oracle
         from paper_2110_04175_gb300 import workloads as wl
 
-        # max over ranks
+        # max / min over ranks
         got = bench.reduce_max(float(rank + 1) * 1.5, world)
         assert got == 1.5 * world
+        assert bench.reduce_min(float(rank + 1) * 1.5, world) == 1.5
         bench.barrier(world)
 
         # d-sharding: each rank runs its slice of a longer vector
