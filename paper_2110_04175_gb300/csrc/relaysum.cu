@@ -2,21 +2,27 @@
 //
 // Vogels et al., "RelaySum for Decentralized Deep Learning on Heterogeneous
 // Data" (arXiv 2110.04175), Algorithm 1 (RelaySGD) with the robust rebuild of
-// Section 4.4, for n virtual workers on one GPU.  See relaysum.h for the
-// equations and the ABI contract, program.h for the visit program.
+// Section 4.4, local momentum / Adam, lost messages, and the appendix's
+// RelaySum/Grad and mean-estimation algorithms on the same relay, for n
+// virtual workers on one GPU.  See relaysum.h for the equations and the ABI
+// contract, program.h for the visit program.
 //
 // Kernels:
-//   relay_counts_kernel   Alg. 1 counters, int32, one CTA, in place.
+//   relay_counts_kernel   Alg. 1 counters, int32, one CTA, in place (lost
+//                         messages count 0; mean estimation's counts s_i).
 //   relay_models_kernel   everything per coordinate, in ONE pass over d:
-//                         local step with Philox noise, every outgoing relay
-//                         message, every rebuild.  Each x_i, mu_i and incoming
-//                         message quad is read from HBM once and each outgoing
-//                         message / new model quad written once (a child of a
-//                         node of degree > 4 re-reads the one message it sent
-//                         that node, see program.h).  The path is bandwidth-bound
-//                         streaming arithmetic: no tensor cores.
+//                         local step (SGD / Nesterov / Adam) with Philox noise,
+//                         every outgoing relay message, every rebuild.  Each
+//                         x_i, mu_i and incoming message quad is read from HBM
+//                         once and each outgoing message / new model quad
+//                         written once (a child of a node of degree > 4
+//                         re-reads the one message it sent that node, see
+//                         program.h).  The path is bandwidth-bound streaming
+//                         arithmetic: no tensor cores.
 //   relay_init_kernel     x^0 (shared Philox draw) and zeroed messages.
 //   relay_fill_mu_kernel  mu_i = scale * sum_k mix[i][k] N_k.
+//   relay_metrics_kernel  consensus distance and distance to the optimum,
+//   (+ _finish_kernel)    two fixed-order passes in double.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -883,12 +889,10 @@ int relay_init(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* c
         return RELAY_ECUDA;
     if (h->d == 0) return RELAY_OK;
     // optimiser state starts at zero (momentum buffer, Adam moments)
-    const size_t state_bytes = static_cast<size_t>((h->prog.n - 1) * h->ld_x + 4 * h->nquads) * 4;
     for (float* st : {h->s1, h->s2})
         if (st && cudaMemset2DAsync(st, static_cast<size_t>(h->ld_x) * 4, 0, static_cast<size_t>(4 * h->nquads) * 4,
                                     static_cast<size_t>(h->prog.n), stream) != cudaSuccess)
             return RELAY_ECUDA;
-    (void)state_bytes;
     const int threads = 256;
     relay_init_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
         x, E > 0 ? msg_a : nullptr, E > 0 ? msg_b : nullptr, h->prog.n, E, h->ld_x, h->ld_m, h->nquads,
