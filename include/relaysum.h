@@ -35,6 +35,11 @@
  *     status; arguments are checked before anything is enqueued, and a
  *     rejected call leaves every buffer untouched.  RELAY_ECUDA reports a
  *     failed launch (cudaGetLastError); no C++ exception crosses the ABI.
+ *   - Handles.  A handle's settings (offset, strides, objective, optimiser,
+ *     lost messages, ...) are copied into each launch's arguments when a
+ *     call enqueues work, so they may be changed between calls without
+ *     waiting for the GPU.  A handle is not safe for concurrent use from
+ *     several host threads; distinct handles are independent.
  *   - Random numbers.  Philox4x32-10 (Salmon et al., SC'11) with key
  *     (seed lo32, seed hi32) and counter (q, row, step, stream) where q is
  *     the ABSOLUTE coordinate quad (c0 + c) / 4; stream 0 = gradient noise
