@@ -26,6 +26,8 @@ from ._native import (RELAY_EINVAL, RELAY_ECUDA, RELAY_ENOMEM, RELAY_ENOTTREE, R
                       relay_step,
                       relay_step_counts, relay_step_models)
 
+from .lr_correction import lr_correction  # noqa: E402
+
 __all__ = [
     "RELAY_OK", "RELAY_EINVAL", "RELAY_ENOTTREE", "RELAY_ECUDA", "RELAY_ENOMEM",
     "RELAY_EUNSUPPORTED", "RELAY_MAX_N", "RELAY_OPT_SGD", "RELAY_OPT_NESTEROV", "RELAY_OPT_ADAM",
@@ -37,5 +39,5 @@ __all__ = [
     "relay_step_models", "relay_step",
     "relay_nbar", "relay_program", "relay_metrics", "relay_metrics_workspace",
     "relay_metrics_static",
-    "relay_error_string",
+    "relay_error_string", "lr_correction",
 ]

@@ -64,3 +64,18 @@ def test_noise_free_runs_converge_linearly(shape, scale):
         run.step(0.3, 0)
     last = run.metrics()[0].cpu().numpy()
     assert last[0] < 1e-9 * first[0] and last[1] < 1e-9 * max(first[1], 1e-30) + 1e-20
+
+
+@pytest.mark.parametrize("shape,n", [("chain", 16), ("binary", 16), ("star", 16), ("torus", 16)])
+def test_lr_correction_matches_oracle(shape, n):
+    from oracle import oracle
+    edges = {"chain": wl.chain(n), "binary": wl.binary_tree(n), "star": wl.star(n),
+             "torus": wl.torus_spanning_tree(4, 4, 0)}[shape]
+    alpha, limits = rs.lr_correction(n, edges, mode=1, device="cuda:0")
+    E = 2 * (n - 1)
+    x, mu = np.zeros((n, 1)), np.ones((n, 1))
+    msg, c = np.zeros((E, 1)), np.zeros(E, np.int32)
+    oracle.run(n, edges, x, mu, msg, c, 1.0, 0.0, 0, 0, 1, 1)
+    oracle.run(n, edges, x, mu, msg, c, 0.0, 0.0, 0, 1, 5000, 1)
+    assert abs(alpha - x[:, 0].mean()) < 1e-5
+    assert 0.0 < alpha < 1.0

@@ -290,3 +290,29 @@ def test_dme_variance_shrinks_like_one_over_samples():
         est = st.x[i] / st.dme_count[i]
         assert abs(est.mean() - 1.0) < 5 * sigma / np.sqrt(st.dme_count[i] * L)
         assert abs(est.var() * st.dme_count[i] / sigma ** 2 - 1.0) < 0.05
+
+
+# ------------------------------------------------ learning-rate correction
+
+def _alpha(n, edges, mode, steps=3000):
+    E = 2 * (n - 1)
+    x = np.zeros((n, 1))
+    mu = np.ones((n, 1))
+    msg = np.zeros((E, 1))
+    c = np.zeros(E, np.int32)
+    oracle.run(n, edges, x, mu, msg, c, 1.0, 0.0, 0, 0, 1, mode)
+    oracle.run(n, edges, x, mu, msg, c, 0.0, 0.0, 0, 1, steps, mode)
+    return x[:, 0]
+
+
+def test_lr_correction_closed_forms():
+    """Algorithm 1's division by nbar loses nothing (alpha = 1 on any tree);
+    so does any rule on n <= 2 (all-reduce from the first step).  Under the
+    robust rule alpha < 1 and is the same on every worker."""
+    for edges in (wl.chain(9), wl.binary_tree(11), wl.star(7), wl.random_tree(12, 3)):
+        n = int(np.max(edges)) + 1
+        assert np.allclose(_alpha(n, edges, 0), 1.0, rtol=0, atol=1e-12)
+        a = _alpha(n, edges, 1)
+        assert 0.0 < a.mean() < 1.0 and np.ptp(a) < 1e-9
+    assert np.allclose(_alpha(2, [(0, 1)], 1), 1.0, atol=1e-12)
+    assert np.allclose(_alpha(1, np.zeros((0, 2), np.int32), 1), 1.0, atol=1e-12)
