@@ -10,7 +10,9 @@ one contiguous block).  A step:
 2. streams the chunks through a ring of device buffers on three CUDA
    streams -- host-to-device copies, the fused kernel (relay_step_models on
    a handle whose coordinate offset is the chunk's absolute position), and
-   device-to-host copies -- so both copy directions and the kernels overlap;
+   device-to-host copies -- so both copy directions and the kernels overlap
+   (message rows arriving at a leaf are never read by the kernel and are not
+   copied in);
 3. copies the counters out.
 
 Ordering: every reuse of a device buffer waits for the copy-out of the chunk
@@ -56,6 +58,22 @@ class HostRelayRun:
         h0 = self.handles[self.widths[0]]
         self.E = nat.relay_num_edges(h0)
         E1 = max(self.E, 1)
+        # message rows the kernel reads: all but those arriving at a leaf (a
+        # leaf's only outgoing message excludes its only incoming one), as
+        # contiguous runs; the others are not copied in (their device rows
+        # are never read)
+        if self.E > 0:
+            _, _, node, pos = nat.relay_program(h0)
+            unread = {int(pos[node[i][1]][0]) for i in range(n) if node[i][0] == 1}
+            rows = [e for e in range(self.E) if e not in unread]
+        else:
+            rows = []
+        self.read_runs = []
+        for e in rows:
+            if self.read_runs and self.read_runs[-1][1] == e:
+                self.read_runs[-1][1] = e + 1
+            else:
+                self.read_runs.append([e, e + 1])
         pin = dict(dtype=torch.float32, pin_memory=True)
         self.x_h = torch.empty(self.nchunks, n, self.cw, **pin)
         self.msg_h = [torch.empty(self.nchunks, E1, self.cw, **pin) for _ in range(2)]
@@ -123,7 +141,8 @@ class HostRelayRun:
                 s_in.wait_event(self.out_done[b])
                 s_in.wait_event(self.out_done_k[k])
                 self.xb[b].copy_(self.x_h[k], non_blocking=True)
-                self.mib[b].copy_(src[k], non_blocking=True)
+                for lo, hi in self.read_runs:
+                    self.mib[b][lo:hi].copy_(src[k][lo:hi], non_blocking=True)
                 self.in_done[b].record(s_in)
             self.s_comp.wait_event(self.in_done[b])
             nat.relay_step_models(self._handle(k), self.xb[b], self.mib[b], self.mob[b],
@@ -148,8 +167,10 @@ class HostRelayRun:
 
     def bytes_per_step(self):
         """(host-to-device, device-to-host) bytes copied per step."""
-        h2d = (self.x_h.numel() + self.msg_h[0].numel() + self.counts_h.numel()) * 4
-        return h2d, h2d
+        rows_in = sum(hi - lo for lo, hi in self.read_runs)
+        h2d = (self.x_h.numel() + self.nchunks * rows_in * self.cw + self.counts_h.numel()) * 4
+        d2h = (self.x_h.numel() + self.msg_h[0].numel() + self.counts_h.numel()) * 4
+        return h2d, d2h
 
     def models(self):
         """x as a host [n][d] array (a copy)."""
