@@ -14,7 +14,8 @@ Prints one JSON line.  `value` is whole-job steps/s with the state resident
 in HBM; `e2e` is the same metric through relay_step with the state in pinned
 host buffers (copies inside the timed region); `roofline` is the fused
 kernel's algorithmic HBM bytes per launch over its CUDA-event duration;
-`cpu_baseline` times the plain CPU oracle on a bounded coordinate sample.
+`cpu_baseline` times the plain CPU oracle on a bounded coordinate sample,
+on every host core (one slice per thread) and on one thread.
 
 Multi-GPU (torchrun, one rank per GPU): every rank runs the same workload on
 its own d-slice of one longer model vector (coordinates are independent, so
@@ -167,61 +168,122 @@ def bus_id_of(device: int) -> str | None:
 
 # -------------------------------------------------------------- CPU oracle
 
-def oracle_sample(w, seconds: float = 15.0, max_len: int = 1 << 20):
-    """Times the oracle (as it stands, one thread) on a coordinate slice of
-    workload `w`, scaled to steps/s of the full d."""
-    import numpy as np
-    from oracle import oracle
-    edges = w.edges[0] if isinstance(w.edges, list) else w.edges  # a sample in the first window
-    length = 2048
-    st = oracle.State(w.n, edges, length)
-    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
-    t0 = time.perf_counter()
-    st.advance(1, w.lr, w.sigma, w.seed, w.mode)
-    per_coord_step = (time.perf_counter() - t0) / length
-    steps = 4
-    length = int(min(max_len, w.d, max(1024, seconds / (steps * per_coord_step))))
-    st = oracle.State(w.n, edges, length)
-    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
-    t0 = time.perf_counter()
-    st.advance(steps, w.lr, w.sigma, w.seed, w.mode)
-    dt = time.perf_counter() - t0
-    return {"value": steps / dt * length / w.d, "unit": "steps/s", "cores": 1, "kind": "oracle",
-            "sample": f"{steps} steps of coordinates [0, {length}) of d = {w.d} "
-                      f"({dt:.1f} s, one thread), scaled by {length}/{w.d}"}
+def host_threads() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+class OracleSlices:
+    """The oracle, as it stands, on `threads` disjoint consecutive coordinate
+    slices of workload `w`, advanced concurrently (each thread one slice; the
+    ctypes calls release the GIL, so the slices run on separate cores)."""
+
+    def __init__(self, w, length: int, threads: int):
+        import numpy as np
+        from oracle import oracle
+        edges = w.edges[0] if isinstance(w.edges, list) else w.edges  # a sample in the first window
+        self.w, self.length, self.threads = w, length, threads
+        self.states = [oracle.State(w.n, edges, length, c0=k * length) for k in range(threads)]
+        self.pool = None
+        if threads > 1:
+            from concurrent.futures import ThreadPoolExecutor
+            self.pool = ThreadPoolExecutor(threads)
+        mix = w.mix.astype(np.float64)
+        self._each(lambda st: st.init(w.x0_std, w.seed, mix, w.mu_scale, w.mu_seed))
+
+    def _each(self, fn):
+        if self.pool is None:
+            fn(self.states[0])
+        else:
+            list(self.pool.map(fn, self.states))
+
+    def advance(self, steps: int) -> float:
+        """Wall-clock seconds for `steps` steps of every slice."""
+        w = self.w
+        t0 = time.perf_counter()
+        self._each(lambda st: st.advance(steps, w.lr, w.sigma, w.seed, w.mode))
+        return time.perf_counter() - t0
+
+    def close(self):
+        if self.pool is not None:
+            self.pool.shutdown()
+
+
+def oracle_bytes_per_coord(w) -> int:
+    """Host bytes one oracle coordinate holds: x, mu, messages and the
+    step's temporaries (x^{t+1/2}, new messages), fp64."""
+    return 8 * (3 * w.n + 2 * 2 * (w.n - 1))
+
+
+def oracle_plan(w, threads: int, mem_per_thread: int):
+    """(threads, coordinates per thread) for a concurrent oracle sample of
+    `w`: at most `mem_per_thread` host bytes per slice, within d."""
+    cap = max(4, mem_per_thread // oracle_bytes_per_coord(w))
+    threads = max(1, min(threads, w.d // 1024))
+    return threads, max(4, min(cap, w.d // threads) // 4 * 4)
+
+
+def oracle_per_coord(w) -> float:
+    """One-thread seconds per coordinate-step of the oracle on `w`."""
+    probe = OracleSlices(w, min(4096, max(4, w.d // 4 * 4)), 1)
+    probe.advance(1)
+    dt = probe.advance(1)
+    return dt / probe.length
+
+
+def oracle_sample(w, seconds: float = 8.0):
+    """Times the oracle (as it stands) on bounded coordinate samples of
+    workload `w`, scaled to steps/s of the full d: on every host core (one
+    slice per thread) and, for reference, on one thread.  The slices are
+    small (the oracle's centre fill costs about as much as 25 steps) and
+    the step counts fill about `seconds` each at one thread's rate."""
+    per_coord = oracle_per_coord(w)
+    threads, lt = oracle_plan(w, host_threads(), 96 << 20)
+    steps = int(max(2, min(200, round(seconds / (lt * per_coord)))))
+    one = OracleSlices(w, lt, 1)
+    steps1 = max(1, steps // 2)
+    dt1 = one.advance(steps1)
+    one.close()
+    del one
+    many = OracleSlices(w, lt, threads)
+    dt = many.advance(steps)
+    many.close()
+    del many
+    return {"value": steps / dt * threads * lt / w.d, "unit": "steps/s", "cores": threads,
+            "kind": "oracle", "value_1thread": steps1 / dt1 * lt / w.d,
+            "sample": f"{steps} steps of coordinates [0, {threads * lt}) of d = {w.d}, "
+                      f"{threads} threads of {lt} coordinates each ({dt:.1f} s), scaled by "
+                      f"{threads * lt}/{w.d}; value_1thread: {steps1} steps of [0, {lt}) on one "
+                      f"thread ({dt1:.1f} s)"}
 
 
 def run_reference(args, w, rank: int):
     """The reference arm: the plain CPU oracle on bounded samples of the
-    same workload; each step is one oracle step over a coordinate slice."""
-    import numpy as np
-    from oracle import oracle
+    same workload; each step is one oracle step over a coordinate slice per
+    host core, run concurrently."""
     if rank != 0:
         return
-    edges = w.edges[0] if isinstance(w.edges, list) else w.edges  # a sample in the first window
-    length = 4096
-    st = oracle.State(w.n, edges, length)
-    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
-    t0 = time.perf_counter()
-    st.advance(1, w.lr, w.sigma, w.seed, w.mode)
-    per_coord = (time.perf_counter() - t0) / length
-    budget = 90.0 / max(1, args.steps + args.warmup)
-    length = int(max(256, min(1 << 20, w.d, budget / per_coord)))
-    st = oracle.State(w.n, edges, length)
-    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
-    st.advance(args.warmup, w.lr, w.sigma, w.seed, w.mode)
-    t0 = time.perf_counter()
-    st.advance(args.steps, w.lr, w.sigma, w.seed, w.mode)
-    dt = time.perf_counter() - t0
+    per_coord = oracle_per_coord(w)
+    budget = 90.0 / max(1, args.steps + args.warmup)  # seconds per step at one thread's rate
+    threads, lt = oracle_plan(w, host_threads(), 192 << 20)
+    lt = max(4, min(lt, int(budget / per_coord)) // 4 * 4)
+    sl = OracleSlices(w, lt, threads)
+    if args.warmup:
+        sl.advance(args.warmup)
+    dt = sl.advance(args.steps)
+    sl.close()
+    length = threads * lt
     value = args.steps / dt * length / w.d
     sample = (f"each step: one oracle step over coordinates [0, {length}) of d = {w.d}, "
-              f"one thread; steps/s scaled by {length}/{w.d}")
+              f"{threads} threads of {lt} coordinates each; steps/s scaled by {length}/{w.d}")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt / args.steps * 1e3 * w.d / length, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(w, args.gpus),
-            "cpu_baseline": {"value": value, "unit": "steps/s", "cores": 1, "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": "steps/s", "cores": threads, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
