@@ -456,6 +456,38 @@ def pinned_like(t):
     return torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
 
 
+def host_link_gbs(dev, mib: int = 1024, reps: int = 4) -> dict:
+    """Measured copy rates of this GPU's host link with pinned memory and the
+    copy engines: host-to-device alone, device-to-host alone, and both at
+    once on two streams (the e2e path's ceiling)."""
+    import torch
+    n = mib << 18  # floats
+    hin = torch.ones(n, dtype=torch.float32, pin_memory=True)
+    hout = torch.empty(n, dtype=torch.float32, pin_memory=True)
+    din = torch.empty(n, dtype=torch.float32, device=dev)
+    dout = torch.zeros(n, dtype=torch.float32, device=dev)
+    s1, s2 = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+
+    def timed(h2d: bool, d2h: bool) -> float:
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            if h2d:
+                with torch.cuda.stream(s1):
+                    din.copy_(hin, non_blocking=True)
+            if d2h:
+                with torch.cuda.stream(s2):
+                    hout.copy_(dout, non_blocking=True)
+        torch.cuda.synchronize(dev)
+        return (int(h2d) + int(d2h)) * reps * n * 4 / (time.perf_counter() - t0) / 1e9
+
+    timed(True, True)  # warm-up
+    out = {"h2d_gbs": timed(True, False), "d2h_gbs": timed(False, True),
+           "both_gbs": timed(True, True)}
+    del hin, hout, din, dout
+    return {k: round(v, 1) for k, v in out.items()}
+
+
 def run_e2e(args, w, run, dev, stream, world: int):
     """The same metric through the host-state API: x, both message buffers and
     the counters live in pinned host memory and every step streams them
@@ -486,6 +518,7 @@ def run_e2e(args, w, run, dev, stream, world: int):
     del run.trees[:]
     run.x = run.mu = None
     torch.cuda.empty_cache()
+    link = host_link_gbs(dev)
     host = HostRelayRun(w.n, w.d, w.edges, chunk=cw, device=dev, mode=w.mode,
                         c0=shard_offset(int(os.environ.get("RANK", "0")), w.d),
                         copy_streams=args.copy_streams)
@@ -504,7 +537,9 @@ def run_e2e(args, w, run, dev, stream, world: int):
             "path": "HostRelayRun: state in pinned host memory, streamed through the GPU in "
                     f"{host.nchunks} chunks of {cw} coordinates ({args.copy_streams} copy-in / "
                     f"kernel / {args.copy_streams} copy-out streams), copies inside the timed region",
-            "copy_gbs": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9, 1)}
+            "copy_gbs": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9, 1),
+            "host_link": link,
+            "copy_frac": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9 / link["both_gbs"], 3)}
 
 
 def traffic_per_launch(w, objective: str):
