@@ -282,7 +282,7 @@ def run_reference(args, w, rank: int):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt / args.steps * 1e3 * w.d / length, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(w, args.gpus),
+            "config": workload_config(w, args.gpus, args),
             "cpu_baseline": {"value": value, "unit": "steps/s", "cores": threads, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0,
@@ -290,7 +290,35 @@ def run_reference(args, w, rank: int):
     print(json.dumps(line), flush=True)
 
 
-def workload_config(w, gpus: int, args=None) -> dict:
+def l2_bytes(dev) -> int:
+    import torch
+    return int(getattr(torch.cuda.get_device_properties(dev), "L2_cache_size", 0) or (129 << 20))
+
+
+def step_bytes(w, args=None) -> int:
+    """HBM bytes one step touches: the algorithmic bytes plus stored centres."""
+    stored = args is None or args.objective == "stored"
+    return w.bytes_per_step() + (4 * w.d * w.n if stored else 0)
+
+
+def l2_flush_needed(w, args, dev) -> bool:
+    if args.l2_flush != "auto":
+        return args.l2_flush == "on"
+    return step_bytes(w, args) < 2 * l2_bytes(dev)
+
+
+def l2_note(w, args, dev=None) -> str:
+    mb = step_bytes(w, args) / 1e6
+    if args is not None and args.graph:
+        return (f"working set {mb:.1f} MB per step; the captured steps run back to back with no "
+                f"L2 flush between them (L2-resident where it fits)")
+    if dev is not None and args is not None and l2_flush_needed(w, args, dev):
+        return (f"working set {mb:.1f} MB per step, under twice the L2: L2 flushed (memset of "
+                f"{2 * l2_bytes(dev) / 1e6:.0f} MB) before every timed step, steps timed one by one")
+    return f"inputs larger than L2 ({mb / 1e3:.1f} GB moved per step)"
+
+
+def workload_config(w, gpus: int, args=None, dev=None) -> dict:
     shape = {"binary": "balanced binary tree (heap order)", "chain": "chain", "star": "star",
              "torus": "uniform spanning tree of the 8x8 torus",
              "double": "double binary trees (two complementary trees, half the coordinates each)"}
@@ -298,7 +326,7 @@ def workload_config(w, gpus: int, args=None) -> dict:
     return {"workload": w.name, "n_workers": w.n, "tree": kind, "d": w.d, "directed_edges": w.E,
             "rebuild": "robust (Section 4.4)" if w.mode == 1 else "Algorithm 1",
             "sigma": w.sigma, "lr": w.lr, "objective": "identity-Hessian heterogeneous quadratics",
-            "l2": f"inputs larger than L2 ({w.bytes_per_step() / 1e9:.1f} GB moved per step)",
+            "l2": l2_note(w, args, dev),
             "parallelism": f"d-sharded over {gpus} rank(s), no collective" if gpus > 1
             else "1 GPU",
             **({"algorithm": args.algorithm, "local_optimizer": args.optimizer,
@@ -321,10 +349,12 @@ def run_native(args, w, rank: int, world: int):
     optimizer = {"sgd": None, "nesterov": ("nesterov", 0.9),
                  "adam": ("adam", 0.9, 0.999, 1e-8)}[args.optimizer]
     run = rs.RelayRun(w.n, w.d, w.edges, device=dev, mode=w.mode, c0=c0, objective=args.objective,
-                      optimizer=optimizer, algorithm=args.algorithm)
+                      optimizer=optimizer, algorithm=args.algorithm, kernel=args.kernel)
     lost_rng = np.random.default_rng(1234 + rank)
     run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
     h = run.h
+    kernel_name = ("relay_nodes_kernel" if rs.relay_get_kernel(h) == rs.RELAY_KERNEL_NODES
+                   else "relay_models_kernel")
 
     def one_step(ev=None):
         for k, tr in enumerate(run.trees):
@@ -347,6 +377,11 @@ def run_native(args, w, rank: int, world: int):
         one_step()
     if args.graph:
         return run_graphed(args, w, run, dev, stream, rank, world)
+    # a working set that fits in L2 is evicted before every timed step (a
+    # memset of twice the L2), and the steps are then timed one by one
+    flush = None
+    if l2_flush_needed(w, args, dev):
+        flush = torch.empty(2 * l2_bytes(dev), dtype=torch.uint8, device=dev)
     events = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(T)]
               for _ in range(args.steps)]
     torch.cuda.synchronize(dev)
@@ -354,11 +389,17 @@ def run_native(args, w, rank: int, world: int):
     torch.cuda.synchronize(dev)
     with ClockSampler(bus_id_of(local) if rank == 0 else None) as clocks:
         for k in range(args.steps):
+            if flush is not None:
+                flush.zero_()
             one_step(events[k])
         torch.cuda.synchronize(dev)
     barrier(world)
     torch.cuda.synchronize(dev)
-    total_ms = events[0][0][0].elapsed_time(events[-1][-1][2])
+    if flush is None:
+        total_ms = events[0][0][0].elapsed_time(events[-1][-1][2])
+    else:
+        total_ms = sum(events[k][0][0].elapsed_time(events[k][-1][2]) for k in range(args.steps))
+        del flush
     # fused-kernel time per step (one launch per tree)
     models_ms = [sum(events[k][j][1].elapsed_time(events[k][j][2]) for j in range(T))
                  for k in range(args.steps)]
@@ -382,8 +423,9 @@ def run_native(args, w, rank: int, world: int):
     moved = alg_bytes if args.objective == "generated" else alg_bytes + 4 * w.d * w.n
     achieved = alg_bytes / (mean_models_ms / 1e3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                "frac": round(achieved / peak, 4), "traffic": traffic_per_launch(w, args.objective),
-                "kernel": "relay_models_kernel", "peak_source": peak_src,
+                "frac": round(achieved / peak, 4),
+                "traffic": traffic_per_launch(w, args.objective, kernel_name),
+                "kernel": kernel_name, "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "algorithmic_bytes_rule": "4 d (2n + 2E) [+ 4 d n x optimiser-state rows]",
                 "objective": args.objective,
@@ -398,7 +440,7 @@ def run_native(args, w, rank: int, world: int):
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": workload_config(w, world, args), "roofline": roofline, "cpu_baseline": cpu,
+            "config": workload_config(w, world, args, dev), "roofline": roofline, "cpu_baseline": cpu,
             "e2e": e2e, "gpu_launches": 2 * T * args.steps, "clocks": clocks.summary(),
             "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1)}
     print(json.dumps(line), flush=True)
@@ -542,16 +584,18 @@ def run_e2e(args, w, run, dev, stream, world: int):
             "copy_frac": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9 / link["both_gbs"], 3)}
 
 
-def traffic_per_launch(w, objective: str):
-    """DRAM bytes per launch of the fused kernel from the committed ncu
-    summary for this workload and objective source (profiles/traffic.txt),
-    or None when no capture of the current kernel exists for it."""
+def traffic_per_launch(w, objective: str, kernel: str = "relay_models_kernel"):
+    """DRAM bytes per launch of the step kernel from the committed ncu
+    summary for this kernel, workload and objective source
+    (profiles/traffic.txt), or None when no capture of the current kernel
+    exists for it."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     try:
         with open(path) as f:
             for line in f:
                 parts = line.split()
-                if len(parts) == 2 and not line.startswith("#") and parts[0] == f"{w.name}/{objective}":
+                if len(parts) == 2 and not line.startswith("#") and \
+                        parts[0] == f"{kernel}/{w.name}/{objective}":
                     return int(parts[1])
     except OSError:
         pass
@@ -569,6 +613,11 @@ def main(argv=None):
     p.add_argument("--copy-streams", type=int, default=2,
                    help="copy streams per direction of the host-state path")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--kernel", choices=["auto", "walk", "nodes"], default="auto",
+                   help="step kernel (relay_set_kernel)")
+    p.add_argument("--l2-flush", choices=["auto", "on", "off"], default="auto",
+                   help="flush L2 before every timed step (auto: when a step's working set is "
+                        "under twice the L2)")
     p.add_argument("--optimizer", choices=["sgd", "nesterov", "adam"], default="sgd",
                    help="local optimiser of the local step (appendix: momentum / Adam)")
     p.add_argument("--algorithm", choices=["relaysgd", "grad", "dme"], default="relaysgd",

@@ -136,6 +136,23 @@ int relay_set_lost_messages(relay_handle *h, const uint8_t *lost);
  * The default is 1. */
 int relay_set_rebuild_mode(relay_handle *h, int32_t mode);
 
+/* Which kernel runs the fused step (an implementation choice: the paper's
+ * Algorithm 1 fixes only what is computed).  RELAY_KERNEL_WALK: one thread
+ * per quad of coordinates walks every worker of the tree in turn.
+ * RELAY_KERNEL_NODES: one thread per (worker, quad), the new messages meeting
+ * in shared memory; it uses n times more threads, which pays off when d is
+ * short.  Both form every sum in the same order, so their results are
+ * identical bit for bit.  RELAY_KERNEL_AUTO (the default) picks by d.
+ * Errors: RELAY_EINVAL for another value. */
+#define RELAY_KERNEL_AUTO 0
+#define RELAY_KERNEL_WALK 1
+#define RELAY_KERNEL_NODES 2
+int relay_set_kernel(relay_handle *h, int32_t kernel);
+
+/* The kernel the next step of this handle launches: RELAY_KERNEL_WALK or
+ * RELAY_KERNEL_NODES (RELAY_KERNEL_AUTO resolved), or RELAY_EINVAL. */
+int relay_get_kernel(const relay_handle *h);
+
 /* Absolute index of this handle's first coordinate within a longer model
  * vector (c0 >= 0, a multiple of 4): the noise of local coordinate c is
  * that of coordinate c0 + c, so a vector split into slices -- across GPUs,

@@ -22,6 +22,9 @@ RELAY_OPT_ADAM = 2
 RELAY_ALGO_RELAYSGD = 0
 RELAY_ALGO_GRAD = 1
 RELAY_ALGO_DME = 2
+RELAY_KERNEL_AUTO = 0
+RELAY_KERNEL_WALK = 1
+RELAY_KERNEL_NODES = 2
 
 _lock = threading.Lock()
 _lib = None
@@ -50,6 +53,8 @@ def _load():
             "relay_num_edges": (i32, [vp]),
             "relay_edges": (ctypes.c_int, [vp, vp, vp]),
             "relay_set_rebuild_mode": (ctypes.c_int, [vp, i32]),
+            "relay_set_kernel": (ctypes.c_int, [vp, i32]),
+            "relay_get_kernel": (ctypes.c_int, [vp]),
             "relay_set_strides": (ctypes.c_int, [vp, i64, i64]),
             "relay_set_local_optimizer": (ctypes.c_int, [vp, i32, f32, f32, f32, vp, vp]),
             "relay_set_lost_messages": (ctypes.c_int, [vp, vp]),
@@ -175,6 +180,16 @@ def relay_edges(h):
 
 def relay_set_rebuild_mode(h, mode: int):
     _check(_load().relay_set_rebuild_mode(_h(h), int(mode)), "relay_set_rebuild_mode")
+
+
+def relay_set_kernel(h, kernel: int):
+    _check(_load().relay_set_kernel(_h(h), int(kernel)), "relay_set_kernel")
+
+
+def relay_get_kernel(h) -> int:
+    k = _load().relay_get_kernel(_h(h))
+    _check(min(k, 0), "relay_get_kernel")
+    return k
 
 
 def relay_set_strides(h, ld_x: int, ld_msg: int):
@@ -313,10 +328,12 @@ class RelayRun:
     """
 
     def __init__(self, n: int, d: int, edges, device="cuda", mode: int = 1, c0: int = 0,
-                 objective: str = "stored", optimizer=None, algorithm: str = "relaysgd"):
+                 objective: str = "stored", optimizer=None, algorithm: str = "relaysgd",
+                 kernel: str = "auto"):
         """optimizer: None (SGD), ("nesterov", beta1) or ("adam", beta1, beta2, eps);
         algorithm: "relaysgd" (Alg. 1), "grad" (Alg. 6) or "dme" (Alg. 5, x holds
-        the running sums y and `dme_count` the counts s of each tree)."""
+        the running sums y and `dme_count` the counts s of each tree);
+        kernel: "auto", "walk" or "nodes" (relay_set_kernel)."""
         import torch
         if objective not in ("stored", "generated"):
             raise ValueError(objective)
@@ -339,6 +356,8 @@ class RelayRun:
             dk = min(4 * q_hi, d) - col0 if q_hi > q_lo else 0
             h = relay_create(n, dk, tree_edges)
             relay_set_rebuild_mode(h, mode)
+            relay_set_kernel(h, {"auto": RELAY_KERNEL_AUTO, "walk": RELAY_KERNEL_WALK,
+                                 "nodes": RELAY_KERNEL_NODES}[kernel])
             relay_set_coord_offset(h, c0 + col0)
             ld_m = relay_ld(h)
             relay_set_strides(h, self.ld, ld_m)

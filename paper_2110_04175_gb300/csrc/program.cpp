@@ -244,6 +244,18 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
         }
         p->order[v] = static_cast<int16_t>(i);
     }
+    // rebuild order of every worker's incoming messages: the walk adds the
+    // DFS parent's message at the worker's visit, then each child's at the
+    // child's visit
+    auto in_from = [&](int i, int k) {
+        const auto& l = t.nbr[i];
+        return t.in_edge[i][std::lower_bound(l.begin(), l.end(), k) - l.begin()];
+    };
+    for (int i = 0; i < n; ++i) {
+        int k = pos_base[i];
+        if (w.parent[i] >= 0) p->rb_in[k++] = static_cast<int16_t>(in_from(i, w.parent[i]));
+        for (int c : w.children[i]) p->rb_in[k++] = static_cast<int16_t>(in_from(i, c));
+    }
     (void)root;
     return next_id;
 }

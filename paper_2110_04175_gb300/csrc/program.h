@@ -21,6 +21,11 @@
 //     message) and writes it out.  This keeps the slots per thread O(1)
 //     instead of O(degree).
 //
+// The same program drives the node-parallel kernel for short vectors (one
+// thread per worker and quad): it forms each worker's messages with the
+// walk's arithmetic and adds the incoming ones in the walk's order (rb_in),
+// so both kernels give the same bits.
+//
 // The program is a plain-old-data struct passed by value as a
 // __grid_constant__ kernel parameter (warp-uniform reads from the constant
 // bank), so a handle owns no device memory.
@@ -60,6 +65,9 @@ struct Program {
     int16_t pos_slot[kMaxE];     // narrow node: slot of the message to child k_s; else -1
     int16_t edge_src[kMaxE];     // directed edge e: edge_src[e] -> edge_dst[e]
     int16_t edge_dst[kMaxE];
+    int16_t rb_in[kMaxE];        // i's positions: its incoming edges in the walk's rebuild
+                                 // order (from the DFS parent, then from the children in
+                                 // visit order); the node-parallel kernel adds them so
 };
 
 // Where the kernel takes the quadratic centres mu_i from.

@@ -19,6 +19,9 @@
 //                         re-reads the one message it sent that node, see
 //                         program.h).  The path is bandwidth-bound streaming
 //                         arithmetic: no tensor cores.
+//   relay_nodes_kernel    the same step for short vectors, one thread per
+//                         (worker, quad) with the new messages exchanged in
+//                         shared memory; same bits as relay_models_kernel.
 //   relay_init_kernel     x^0 (shared Philox draw) and zeroed messages.
 //   relay_fill_mu_kernel  mu_i = scale * sum_k mix[i][k] N_k.
 //   relay_metrics_kernel  consensus distance and distance to the optimum,
@@ -59,6 +62,8 @@ struct relay_handle {
     // algorithm on the relay: 0 RelaySGD (Alg. 1), 1 RelaySum/Grad (Alg. 6), 2 DME (Alg. 5)
     int32_t algo = 0;
     int64_t* dme_count = nullptr;  // algo 2: s_i, device int64 [n]
+    // step kernel: RELAY_KERNEL_AUTO / _WALK / _NODES
+    int32_t kernel = RELAY_KERNEL_AUTO;
     // messages lost in transit (Section 4.4), one bit per directed edge
     bool has_lost = false;
     uint32_t lost[relaysum::kMaxE / 32 + 1] = {};
@@ -365,17 +370,12 @@ __device__ __forceinline__ float4 centre(const Objective& obj, const PhiloxKey& 
     return scale4_rn(acc, obj.scale);
 }
 
-// mode 0: x' = acc / nbar (Alg. 1).  mode 1: x' = (acc + (n - nbar) x) / n
-// (robust rule), with the fill term folded into the accumulator up front.
-// OBJ: where mu comes from (ObjectiveSource).  OPT: the local optimiser
-// (0 SGD, 1 Nesterov momentum, 2 Adam).
-template <int OBJ, int OPT>
-__global__ void __launch_bounds__(128)
-relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant__ Objective obj,
-                    const __grid_constant__ PhiloxKey mu_key, const __grid_constant__ ModelArgs a) {
-    extern __shared__ float4 slot_mem[];
-    __shared__ float s_scale[kMaxN];
-    __shared__ float s_fill[kMaxN];
+// Per-worker rebuild factors from this step's counters: x' = scale * acc
+// with acc = fill * x + x^{t+1/2} + incoming messages.
+//   mode 0: x' = acc / nbar (Alg. 1).  mode 1: x' = (acc + (n - nbar) x) / n
+//   (robust rule), the fill term folded into the accumulator up front.
+__device__ __forceinline__ void rebuild_factors(const Program& prog, const ModelArgs& a, float* s_scale,
+                                                float* s_fill) {
     const int n = prog.n;
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
         const NodeRec r = prog.node[i];
@@ -395,6 +395,34 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
             s_fill[i] = static_cast<float>(n - nbar);
         }
     }
+}
+
+// The relayed value of worker i at quad q: x^{t+1/2} = x + u (Alg. 1), the
+// update u (Alg. 6) or the sample mu + sigma xi (Alg. 5), with
+// g = (x - mu) + sigma xi and z the worker's noise normals.
+template <int OPT>
+__device__ __forceinline__ float4 relayed_value(const ModelArgs& a, int i, int64_t q, float4 xv, float4 mv,
+                                                float4 z) {
+    if (a.algo == 2)
+        return make_float4(fmaf(a.sigma, z.x, mv.x), fmaf(a.sigma, z.y, mv.y), fmaf(a.sigma, z.z, mv.z),
+                           fmaf(a.sigma, z.w, mv.w));
+    const float4 g = make_float4(fmaf(a.sigma, z.x, xv.x - mv.x), fmaf(a.sigma, z.y, xv.y - mv.y),
+                                 fmaf(a.sigma, z.z, xv.z - mv.z), fmaf(a.sigma, z.w, xv.w - mv.w));
+    const float4 u = local_update<OPT>(a, i, q, g);
+    return (a.algo == 1) ? u : add4(xv, u);
+}
+
+// OBJ: where mu comes from (ObjectiveSource).  OPT: the local optimiser
+// (0 SGD, 1 Nesterov momentum, 2 Adam).
+template <int OBJ, int OPT>
+__global__ void __launch_bounds__(128)
+relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant__ Objective obj,
+                    const __grid_constant__ PhiloxKey mu_key, const __grid_constant__ ModelArgs a) {
+    extern __shared__ float4 slot_mem[];
+    __shared__ float s_scale[kMaxN];
+    __shared__ float s_fill[kMaxN];
+    const int n = prog.n;
+    rebuild_factors(prog, a, s_scale, s_fill);
     __syncthreads();
     const Slots sl{slot_mem + threadIdx.x, static_cast<int>(blockDim.x)};
     float4* cen = slot_mem + prog.nslots * blockDim.x + threadIdx.x;  // OBJ == kMuCachedCentres
@@ -424,19 +452,7 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
             }
             const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i),
                                      a.step, 0u, a.key);
-            // the relayed value: x^{t+1/2} = x + u (Alg. 1), the update u
-            // (Alg. 6) or the sample mu + sigma xi (Alg. 5), with
-            // g = (x - mu) + sigma xi
-            float4 xh;
-            if (a.algo == 2) {
-                xh = make_float4(fmaf(a.sigma, z.x, mv.x), fmaf(a.sigma, z.y, mv.y), fmaf(a.sigma, z.z, mv.z),
-                                 fmaf(a.sigma, z.w, mv.w));
-            } else {
-                const float4 g = make_float4(fmaf(a.sigma, z.x, xv.x - mv.x), fmaf(a.sigma, z.y, xv.y - mv.y),
-                                             fmaf(a.sigma, z.z, xv.z - mv.z), fmaf(a.sigma, z.w, xv.w - mv.w));
-                const float4 u = local_update<OPT>(a, i, q, g);
-                xh = (a.algo == 1) ? u : add4(xv, u);
-            }
+            const float4 xh = relayed_value<OPT>(a, i, q, xv, mv, z);
             // the rebuild sum starts from fill_i x_i (robust rule: n - nbar_i;
             // Alg. 6: n; Alg. 5: 1; Alg. 1: nothing)
             float4 acc = xh;
@@ -467,6 +483,116 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
                 sl[r.acc_slot] = acc;
             }
         }
+    }
+}
+
+// ------------------------------------------------- node-parallel fused step
+
+// For short vectors the walk leaves the GPU idle (one thread per quad walks
+// all n workers in turn), so this form of the same step gives each
+// (worker, quad) pair its own thread.  A CTA owns qb consecutive quads of
+// every worker (threads worker-major: a worker's qb quads are contiguous).
+// Phase 1: each thread forms x_i^{t+1/2} and worker i's outgoing messages
+// with the walk's arithmetic (prefix + suffix at degree <= kRegDeg, the
+// total minus the reverse message above it), writes them out and leaves
+// them in shared memory.  Phase 2, after one barrier: each thread adds its
+// worker's incoming messages in the walk's order (Program::rb_in) and
+// writes the new model.  The results equal relay_models_kernel's bit for
+// bit, and every array is still read and written once.
+
+// Degree D <= kRegDeg: outgoing message s = prefix(s) + suffix(s+1).
+template <int D>
+__device__ __forceinline__ void node_small(const Program& prog, const NodeRec& r, const ModelArgs& a,
+                                           int64_t q, float4 xh, float4* m_new, int qb) {
+    float4 m[D];
+#pragma unroll
+    for (int s = 0; s < D; ++s) m[s] = ld_stream(a.msg_in + prog.pos_in[r.pos_base + s] * a.ld_m + 4 * q);
+    float4 pre[D];
+    pre[0] = xh;
+#pragma unroll
+    for (int s = 1; s < D; ++s) pre[s] = add4(pre[s - 1], m[s - 1]);
+    float4 suf[D];
+    suf[D - 1] = m[D - 1];
+#pragma unroll
+    for (int s = D - 2; s >= 0; --s) suf[s] = add4(m[s], suf[s + 1]);
+#pragma unroll
+    for (int s = 0; s < D; ++s) {
+        const int e = prog.pos_out[r.pos_base + s];
+        const float4 out = delivered(a, e, (s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]));
+        st_stream(a.msg_out + e * a.ld_m + 4 * q, out);
+        m_new[e * qb] = out;
+    }
+}
+
+// Degree D > kRegDeg: T = x^{t+1/2} + the incoming messages summed over
+// descending positions, then message s = T - (incoming message s), as in
+// visit_wide and at the wide node's children.  The incoming messages wait
+// in shared memory (rows of worker i's own incoming edges).
+__device__ __noinline__ void node_wide(const Program& prog, const NodeRec& r, const ModelArgs& a, int64_t q,
+                                       float4 xh, float4* m_new, float4* m_old, int qb) {
+    const int D = r.deg;
+    const int base = r.pos_base;
+    float4 total = xh;
+    for (int s = D - 1; s >= 0; --s) {
+        const int ein = prog.pos_in[base + s];
+        const float4 m = ld_stream(a.msg_in + ein * a.ld_m + 4 * q);
+        total = add4(total, m);
+        m_old[ein * qb] = m;
+    }
+    for (int s = 0; s < D; ++s) {
+        const int e = prog.pos_out[base + s];
+        const float4 out = delivered(a, e, sub4(total, m_old[prog.pos_in[base + s] * qb]));
+        st_stream(a.msg_out + e * a.ld_m + 4 * q, out);
+        m_new[e * qb] = out;
+    }
+}
+
+// blockDim.x = qb * n <= 1024; dynamic shared memory 2 * E * qb float4.
+template <int OBJ, int OPT>
+__global__ void __launch_bounds__(1024)
+relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__ Objective obj,
+                   const __grid_constant__ PhiloxKey mu_key, const __grid_constant__ ModelArgs a, int qb) {
+    extern __shared__ float4 node_mem[];
+    __shared__ float s_scale[kMaxN];
+    __shared__ float s_fill[kMaxN];
+    // regenerated centres are formed per row (the walk's cached centres are
+    // the same normals mixed in the same order)
+    constexpr int kObj = (OBJ == relaysum::kMuStored) ? relaysum::kMuStored : relaysum::kMuPerRow;
+    rebuild_factors(prog, a, s_scale, s_fill);
+    __syncthreads();
+    const int i = static_cast<int>(threadIdx.x) / qb;
+    const int qi = static_cast<int>(threadIdx.x) - i * qb;
+    float4* m_new = node_mem + qi;                 // m_new[e * qb]: m^t on edge e
+    float4* m_old = node_mem + prog.E * qb + qi;   // m_old[e * qb]: m^{t-1} (wide nodes)
+    const NodeRec r = prog.node[i];
+    const int64_t nblk = (a.nquads + qb - 1) / qb;
+    for (int64_t b = blockIdx.x; b < nblk; b += gridDim.x) {
+        const int64_t q = b * qb + qi;
+        const bool active = q < a.nquads;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (active) {
+            const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
+            const float4 mv = centre<kObj>(obj, mu_key, a, i, q, nullptr, 0);
+            const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i), a.step, 0u,
+                                     a.key);
+            const float4 xh = relayed_value<OPT>(a, i, q, xv, mv, z);
+            acc = xh;
+            if (s_fill[i] != 0.0f) acc = add4(scale4(xv, s_fill[i]), xh);
+            switch (r.deg) {
+                case 0: break;
+                case 1: node_small<1>(prog, r, a, q, xh, m_new, qb); break;
+                case 2: node_small<2>(prog, r, a, q, xh, m_new, qb); break;
+                case 3: node_small<3>(prog, r, a, q, xh, m_new, qb); break;
+                case 4: node_small<4>(prog, r, a, q, xh, m_new, qb); break;
+                default: node_wide(prog, r, a, q, xh, m_new, m_old, qb); break;
+            }
+        }
+        __syncthreads();
+        if (active) {
+            for (int k = 0; k < r.deg; ++k) acc = add4(acc, m_new[prog.rb_in[r.pos_base + k] * qb]);
+            st_stream(a.x + i * a.ld_x + 4 * q, scale4(acc, s_scale[i]));
+        }
+        __syncthreads();  // the next block's phase 1 rewrites m_new
     }
 }
 
@@ -619,6 +745,14 @@ int launch_status() {
     return cudaGetLastError() == cudaSuccess ? RELAY_OK : RELAY_ECUDA;
 }
 
+// AUTO picks the node-parallel kernel below this many quads when no worker
+// has more than kRegDeg neighbours.  Measured on one GB300 (whole step, L2
+// flushed): the node kernel is 1.4-5.4x faster up to 16K quads on chains,
+// binary trees and the torus tree, even at 64K quads and slower above; on
+// a star one thread carries the hub's edges while its CTA waits, so the
+// walk stays faster there beyond a few thousand quads.
+constexpr int64_t kNodesBelowQuads = 32768;
+
 // Threads per CTA for the fused kernel: 128, fewer when the slots would not
 // fit in shared memory.
 int models_threads(int nslots) {
@@ -668,8 +802,67 @@ int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream
     return launch_status();
 }
 
+// Quads per CTA of the node-parallel kernel, threads = qb * n <= 1024: a
+// whole warp per worker up to n = 16 (every per-worker table read is then
+// warp-uniform), half a warp up to 64, then 8 and 4 quads.
+int nodes_qb(int n) { return n <= 16 ? 32 : n <= 64 ? 16 : n <= 128 ? 8 : 4; }
+
+template <int OBJ, int OPT>
+int launch_nodes(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
+    int dev = 0;
+    const int sms = device_sms(&dev);
+    if (sms <= 0) return RELAY_ECUDA;
+    const int qb = nodes_qb(h->prog.n);
+    const int threads = qb * h->prog.n;
+    const size_t smem = static_cast<size_t>(2) * h->prog.E * qb * 16;
+    if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
+    static std::atomic<bool> smem_set[kMaxDevices];
+    if ((dev >= kMaxDevices || !smem_set[dev].load())) {
+        if (cudaFuncSetAttribute(relay_nodes_kernel<OBJ, OPT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kMaxSmem) != cudaSuccess)
+            return RELAY_ECUDA;
+        if (dev < kMaxDevices) smem_set[dev].store(true);
+    }
+    // resident CTAs per SM, cached per device (threads and smem depend on n only)
+    static std::atomic<int64_t> occ_cache[kMaxDevices];
+    int per_sm = 0;
+    const int64_t key = static_cast<int64_t>(smem) * 1024 + threads;
+    const int64_t cached = dev < kMaxDevices ? occ_cache[dev].load() : 0;
+    if (cached != 0 && (cached >> 8) == key) {
+        per_sm = static_cast<int>(cached & 0xFF);
+    } else {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_nodes_kernel<OBJ, OPT>, threads,
+                                                          smem) != cudaSuccess ||
+            per_sm <= 0)
+            return RELAY_ECUDA;
+        if (dev < kMaxDevices) occ_cache[dev].store((key << 8) | (per_sm & 0xFF));
+    }
+    const int64_t want = (a.nquads + qb - 1) / qb;
+    const int64_t cap = static_cast<int64_t>(sms) * per_sm;
+    const int grid = static_cast<int>(want < cap ? want : cap);
+    const PhiloxKey mu_key = philox_key(static_cast<uint64_t>(h->obj.k0) | (static_cast<uint64_t>(h->obj.k1) << 32));
+    relay_nodes_kernel<OBJ, OPT><<<grid, threads, smem, stream>>>(h->prog, h->obj, mu_key, a, qb);
+    return launch_status();
+}
+
+// AUTO: the walk keeps every array's traffic at one pass with one thread
+// per quad; below about one resident wave of those threads the GPU idles,
+// and the node-parallel form (n threads per quad) is used instead.
+bool use_nodes(const relay_handle* h) {
+    if (h->kernel == RELAY_KERNEL_NODES) return true;
+    if (h->kernel == RELAY_KERNEL_WALK) return false;
+    if (h->nquads >= kNodesBelowQuads) return false;
+    for (int i = 0; i < h->prog.n; ++i)
+        if (h->prog.node[i].deg > kRegDeg) return false;
+    return true;
+}
+
 template <int OPT>
 int launch_models_obj(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
+    if (use_nodes(h)) {
+        if (h->obj.source == relaysum::kMuStored) return launch_nodes<relaysum::kMuStored, OPT>(h, a, stream);
+        return launch_nodes<relaysum::kMuPerRow, OPT>(h, a, stream);
+    }
     switch (h->obj.source) {
         case relaysum::kMuStored: return launch_models<relaysum::kMuStored, OPT>(h, a, stream);
         case relaysum::kMuPerRow: return launch_models<relaysum::kMuPerRow, OPT>(h, a, stream);
@@ -807,6 +1000,17 @@ int relay_set_rebuild_mode(relay_handle* h, int32_t mode) {
     if (!h || (mode != 0 && mode != 1)) return RELAY_EINVAL;
     h->mode = mode;
     return RELAY_OK;
+}
+
+int relay_set_kernel(relay_handle* h, int32_t kernel) {
+    if (!h || kernel < RELAY_KERNEL_AUTO || kernel > RELAY_KERNEL_NODES) return RELAY_EINVAL;
+    h->kernel = kernel;
+    return RELAY_OK;
+}
+
+int relay_get_kernel(const relay_handle* h) {
+    if (!h) return RELAY_EINVAL;
+    return use_nodes(h) ? RELAY_KERNEL_NODES : RELAY_KERNEL_WALK;
 }
 
 int relay_set_coord_offset(relay_handle* h, int64_t c0) {

@@ -31,10 +31,11 @@ def parity_error(g: np.ndarray, r: np.ndarray) -> float:
 
 
 def gpu_run(w, steps: int, mode: int | None = None, d: int | None = None, c0: int = 0,
-            stream=None, objective: str = "generated") -> rs.RelayRun:
+            stream=None, objective: str = "generated", kernel: str = "auto") -> rs.RelayRun:
     """Runs `steps` RelaySGD steps of workload `w` on cuda:0 through the C ABI."""
     run = rs.RelayRun(w.n, w.d if d is None else d, w.edges, device="cuda:0",
-                      mode=w.mode if mode is None else mode, c0=c0, objective=objective)
+                      mode=w.mode if mode is None else mode, c0=c0, objective=objective,
+                      kernel=kernel)
     run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
     for _ in range(steps):
         run.step(w.lr, w.seed, stream)

@@ -197,3 +197,60 @@ def test_other_algorithms_full_size_sampled(algorithm):
     del run
     gc.collect()
     torch.cuda.empty_cache()
+
+
+# ------------------------------------------------ double binary trees x extensions
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("optimizer,algorithm,lost_p", [
+    ("nesterov", "relaysgd", 0.0), ("adam", "relaysgd", 0.15), (None, "relaysgd", 0.15),
+    ("nesterov", "relaysgd", 0.15), (None, "grad", 0.15), (None, "dme", 0.15)])
+def test_double_binary_trees_with_extensions(optimizer, algorithm, lost_p, mode):
+    """Double binary trees (Section 3) combined with a local optimiser, lost
+    messages (independent masks per tree) and the other algorithms: each
+    tree's coordinate window equals an oracle run of that tree on those
+    coordinates, with its optimiser state, counters and DME counts."""
+    n, d, steps = 16, 2053, 30
+    trees = wl.double_binary_trees(n)
+    run = rs.RelayRun(n, d, list(trees), device="cuda:0", mode=mode, algorithm=algorithm,
+                      optimizer=OPTS[optimizer][1] if optimizer else None)
+    w = wl.Workload("dbt", n, trees[0], d, wl.identity_mix(n), 1.0, 0.1, 0.05, 0.1, steps)
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    if algorithm == "dme":
+        run.x.zero_()
+    E = 2 * (n - 1)
+    rng = np.random.default_rng(11)
+    lost = [(rng.random((steps, E)) < lost_p).astype(np.uint8) for _ in trees]
+    kw = {}
+    if optimizer:
+        o = OPTS[optimizer]
+        kw = dict(opt=o[0], beta1=o[1][1], beta2=o[1][2] if len(o[1]) > 2 else 0.0,
+                  eps=o[1][3] if len(o[1]) > 3 else 0.0)
+    states = []
+    for tr, edges in zip(run.trees, trees):
+        st = oracle.State(n, edges, tr.d, c0=tr.col0)
+        st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+        if algorithm == "dme":
+            st.x[:] = 0.0
+        states.append(st)
+    for t in range(steps):
+        if lost_p > 0:
+            for k in range(len(trees)):
+                run.set_lost(lost[k][t], tree=k)
+        run.step(w.lr, w.seed)
+        for k, st in enumerate(states):
+            st.advance(1, float(np.float32(w.lr)), float(np.float32(w.sigma)), w.seed, mode,
+                       drop=lost[k][t:t + 1] if lost_p > 0 else None,
+                       algo={"relaysgd": oracle.ALGO_RELAYSGD, **ALGOS}[algorithm], **kw)
+    torch.cuda.synchronize()
+    for tr, st in zip(run.trees, states):
+        gx = run.x[:, tr.col0:tr.col0 + tr.d].double().cpu().numpy()
+        gm = tr.messages[:tr.E, :tr.d].double().cpu().numpy()
+        assert parity_error(gx, st.x) <= RTOL, parity_error(gx, st.x)
+        assert parity_error(gm, st.msg) <= RTOL, parity_error(gm, st.msg)
+        assert np.array_equal(tr.counts[:tr.E].cpu().numpy(), st.counts)
+        if algorithm == "dme":
+            assert np.array_equal(tr.dme_count.cpu().numpy(), st.dme_count)
+    del run
+    gc.collect()
+    torch.cuda.empty_cache()

@@ -109,11 +109,12 @@ def test_counts_bit_exact_workload_trees(w):
 
 # ------------------------------------------------------- full-vector parity
 
+@pytest.mark.parametrize("kernel", ["walk", "nodes"])
 @pytest.mark.parametrize("mode", [0, 1])
-def test_chain8_d4096_full_100_steps(mode):
-    """The small workload, every coordinate, 100 steps."""
+def test_chain8_d4096_full_100_steps(mode, kernel):
+    """The small workload, every coordinate, 100 steps, on each step kernel."""
     w = wl.chain8_d4096()
-    run = gpu_run(w, w.steps, mode)
+    run = gpu_run(w, w.steps, mode, kernel=kernel)
     ex, em = compare_ranges(run, w, [(0, w.d)], w.steps, mode)
     assert ex <= RTOL and em <= RTOL, (ex, em)
 
@@ -125,14 +126,16 @@ def test_chain8_d4096_full_100_steps(mode):
     ("star", 9, 131), ("star", 33, 257), ("random", 23, 1031), ("torus", 16, 4099),
     ("star", 256, 67), ("chain", 256, 9),
 ])
-def test_small_cases_every_coordinate(shape, n, d, mode, objective):
+@pytest.mark.parametrize("kernel", ["walk", "nodes"])
+def test_small_cases_every_coordinate(shape, n, d, mode, objective, kernel):
     """Edge cases: one worker, one edge, d below one quad, ragged tails, the
-    generic high-degree path (stars), the largest supported tree."""
+    generic high-degree path (stars), the largest supported tree; on each
+    step kernel."""
     edges = {"single": np.zeros((0, 2), np.int32), "pair": wl.chain(2), "chain": wl.chain(n),
              "binary": wl.binary_tree(n), "star": wl.star(n), "random": wl.random_tree(n, 4),
              "torus": wl.torus_spanning_tree(4, 4, 2)}[shape]
     w = wl.Workload(f"{shape}{n}", n, edges, d, wl.identity_mix(n), 1.0, 0.1, 0.1, 0.1, 30)
-    run = gpu_run(w, w.steps, mode, objective=objective)
+    run = gpu_run(w, w.steps, mode, objective=objective, kernel=kernel)
     ex, em = compare_ranges(run, w, [(0, d)], w.steps, mode)
     assert ex <= RTOL and em <= RTOL, (ex, em)
 

@@ -238,6 +238,15 @@ def test_create_limits_and_layout():
     h = rs.relay_create(3, 8, [(0, 1), (1, 2)])
     with pytest.raises(rs.RelayError):
         rs.relay_set_rebuild_mode(h, 2)
+    for k in (rs.RELAY_KERNEL_WALK, rs.RELAY_KERNEL_NODES):
+        rs.relay_set_kernel(h, k)
+        assert rs.relay_get_kernel(h) == k
+    rs.relay_set_kernel(h, rs.RELAY_KERNEL_AUTO)
+    assert rs.relay_get_kernel(h) in (rs.RELAY_KERNEL_WALK, rs.RELAY_KERNEL_NODES)
+    for k in (-1, 3):
+        with pytest.raises(rs.RelayError) as e:
+            rs.relay_set_kernel(h, k)
+        assert e.value.status == rs.RELAY_EINVAL
     with pytest.raises(rs.RelayError):
         rs.relay_set_coord_offset(h, 6)
     rs.relay_set_coord_offset(h, 8)
