@@ -142,8 +142,9 @@ int relay_set_rebuild_mode(relay_handle *h, int32_t mode);
  * RELAY_KERNEL_NODES: one thread per (worker, quad), the new messages meeting
  * in shared memory; it uses n times more threads, which pays off when d is
  * short.  Both form every sum in the same order, so their results are
- * identical bit for bit.  RELAY_KERNEL_AUTO (the default) picks by d.
- * Errors: RELAY_EINVAL for another value. */
+ * identical bit for bit.  RELAY_KERNEL_AUTO (the default) takes NODES when
+ * n * ceil(d/4) < 2^21 and no worker has more than 4 neighbours (where it
+ * measured faster), WALK otherwise.  Errors: RELAY_EINVAL for another value. */
 #define RELAY_KERNEL_AUTO 0
 #define RELAY_KERNEL_WALK 1
 #define RELAY_KERNEL_NODES 2

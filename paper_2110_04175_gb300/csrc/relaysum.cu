@@ -547,7 +547,12 @@ __device__ __noinline__ void node_wide(const Program& prog, const NodeRec& r, co
     }
 }
 
-// blockDim.x = qb * n <= 1024; dynamic shared memory 2 * E * qb float4.
+// blockDim.x = qb * n <= 1024.  Dynamic shared memory: two [E][qb] float4
+// message buffers used by alternate blocks, plus one more for the incoming
+// messages of wide nodes when the tree has any.  With two buffers a block
+// needs one barrier: a warp already in the next block's phase 1 writes the
+// other buffer, and it can reach this buffer again only after every warp
+// has passed the next block's barrier, i.e. finished reading this one.
 template <int OBJ, int OPT>
 __global__ void __launch_bounds__(1024)
 relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__ Objective obj,
@@ -562,17 +567,34 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
     __syncthreads();
     const int i = static_cast<int>(threadIdx.x) / qb;
     const int qi = static_cast<int>(threadIdx.x) - i * qb;
-    float4* m_new = node_mem + qi;                 // m_new[e * qb]: m^t on edge e
-    float4* m_old = node_mem + prog.E * qb + qi;   // m_old[e * qb]: m^{t-1} (wide nodes)
+    float4* const buf0 = node_mem + qi;                     // [e * qb]: m^t on edge e (even blocks)
+    float4* const buf1 = node_mem + prog.E * qb + qi;       // (odd blocks)
+    float4* const m_old = node_mem + 2 * prog.E * qb + qi;  // [e * qb]: m^{t-1} (wide nodes)
     const NodeRec r = prog.node[i];
+    const float* const xrow = a.x + i * a.ld_x;
+    const float* const murow = a.mu + i * a.ld_x;  // read only for a stored mu
     const int64_t nblk = (a.nquads + qb - 1) / qb;
-    for (int64_t b = blockIdx.x; b < nblk; b += gridDim.x) {
-        const int64_t q = b * qb + qi;
+    const int64_t qstep = static_cast<int64_t>(gridDim.x) * qb;
+    // x (and a stored mu) of this thread's next block are loaded one block
+    // early, so their latency overlaps the barrier and the rebuild
+    float4 xn = make_float4(0.f, 0.f, 0.f, 0.f), mn = xn;
+    int64_t q = static_cast<int64_t>(blockIdx.x) * qb + qi;
+    if (q < a.nquads) {
+        xn = *reinterpret_cast<const float4*>(xrow + 4 * q);
+        if (OBJ == relaysum::kMuStored) mn = ld_stream(murow + 4 * q);
+    }
+    int parity = 0;
+    for (int64_t b = blockIdx.x; b < nblk; b += gridDim.x, q += qstep, parity ^= 1) {
+        float4* const m_new = parity ? buf1 : buf0;
         const bool active = q < a.nquads;
+        const float4 xv = xn, ms = mn;
+        if (q + qstep < a.nquads) {
+            xn = *reinterpret_cast<const float4*>(xrow + 4 * (q + qstep));
+            if (OBJ == relaysum::kMuStored) mn = ld_stream(murow + 4 * (q + qstep));
+        }
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         if (active) {
-            const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
-            const float4 mv = centre<kObj>(obj, mu_key, a, i, q, nullptr, 0);
+            const float4 mv = (OBJ == relaysum::kMuStored) ? ms : centre<kObj>(obj, mu_key, a, i, q, nullptr, 0);
             const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i), a.step, 0u,
                                      a.key);
             const float4 xh = relayed_value<OPT>(a, i, q, xv, mv, z);
@@ -592,7 +614,6 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
             for (int k = 0; k < r.deg; ++k) acc = add4(acc, m_new[prog.rb_in[r.pos_base + k] * qb]);
             st_stream(a.x + i * a.ld_x + 4 * q, scale4(acc, s_scale[i]));
         }
-        __syncthreads();  // the next block's phase 1 rewrites m_new
     }
 }
 
@@ -745,13 +766,13 @@ int launch_status() {
     return cudaGetLastError() == cudaSuccess ? RELAY_OK : RELAY_ECUDA;
 }
 
-// AUTO picks the node-parallel kernel below this many quads when no worker
-// has more than kRegDeg neighbours.  Measured on one GB300 (whole step, L2
-// flushed): the node kernel is 1.4-5.4x faster up to 16K quads on chains,
-// binary trees and the torus tree, even at 64K quads and slower above; on
-// a star one thread carries the hub's edges while its CTA waits, so the
-// walk stays faster there beyond a few thousand quads.
-constexpr int64_t kNodesBelowQuads = 32768;
+// AUTO picks the node-parallel kernel below this many worker-quads (n times
+// the quads) when no worker has more than kRegDeg neighbours.  Measured on
+// one GB300 (whole step, L2 flushed, n = 8 to 64): the node kernel is ahead
+// below about 2^21 worker-quads on chains, binary trees and the torus tree
+// and even or behind above; on a star one thread carries the hub's edges
+// while its CTA waits, so the walk stays faster there.
+constexpr int64_t kNodesBelowWorkerQuads = int64_t(1) << 21;
 
 // Threads per CTA for the fused kernel: 128, fewer when the slots would not
 // fit in shared memory.
@@ -814,7 +835,9 @@ int launch_nodes(const relay_handle* h, const ModelArgs& a, cudaStream_t stream)
     if (sms <= 0) return RELAY_ECUDA;
     const int qb = nodes_qb(h->prog.n);
     const int threads = qb * h->prog.n;
-    const size_t smem = static_cast<size_t>(2) * h->prog.E * qb * 16;
+    bool wide = false;
+    for (int i = 0; i < h->prog.n; ++i) wide = wide || h->prog.node[i].deg > kRegDeg;
+    const size_t smem = static_cast<size_t>(wide ? 3 : 2) * h->prog.E * qb * 16;
     if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
     static std::atomic<bool> smem_set[kMaxDevices];
     if ((dev >= kMaxDevices || !smem_set[dev].load())) {
@@ -851,7 +874,7 @@ int launch_nodes(const relay_handle* h, const ModelArgs& a, cudaStream_t stream)
 bool use_nodes(const relay_handle* h) {
     if (h->kernel == RELAY_KERNEL_NODES) return true;
     if (h->kernel == RELAY_KERNEL_WALK) return false;
-    if (h->nquads >= kNodesBelowQuads) return false;
+    if (h->nquads * h->prog.n >= kNodesBelowWorkerQuads) return false;
     for (int i = 0; i < h->prog.n; ++i)
         if (h->prog.node[i].deg > kRegDeg) return false;
     return true;
