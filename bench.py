@@ -40,6 +40,7 @@ if ROOT not in sys.path:
 METRIC = "RelaySum steps/s and achieved HBM GB/s (fraction of GB300 peak) vs CPU oracle"
 DEFAULT_WORKLOAD = "binary32_d110000000"
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e, nominal
 
 
 # ------------------------------------------------------------ host helpers
@@ -432,7 +433,13 @@ def run_native(args, w, rank: int, world: int):
                 "design_bytes_per_launch": moved,
                 "achieved_design_bytes": round(moved / (mean_models_ms / 1e3) / 1e9, 1),
                 "launch_ms_mean": round(mean_models_ms, 4),
-                "launch_ms_min": round(min(models_ms), 4)}
+                "launch_ms_min": round(min(models_ms), 4),
+                "nominal_peak": NOMINAL_HBM_GBS,
+                "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4)}
+    if roofline["traffic"]:
+        # the ncu DRAM bytes of one launch over this run's mean launch time
+        roofline["dram_gbs"] = round(roofline["traffic"] / (mean_models_ms / 1e3) / 1e9, 1)
+        roofline["dram_frac"] = round(roofline["dram_gbs"] / peak, 4)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         cpu = oracle_sample(w)
