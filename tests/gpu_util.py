@@ -11,6 +11,8 @@ and its fp32 logf/sincospif in the noise.
 """
 from __future__ import annotations
 
+import os
+
 import numpy as np
 import torch
 
@@ -51,6 +53,23 @@ def oracle_range(w, c0: int, length: int, steps: int, mode: int | None = None) -
     return st
 
 
+def windows(d: int, width: int = 16384):
+    """Every coordinate of [0, d) as consecutive windows (parallel oracle work)."""
+    return [(s, min(width, d - s)) for s in range(0, d, width)]
+
+
+def c8_sample(d: int, seed: int, edge: int = 65536, n_windows: int = 1024, width: int = 1024):
+    """The full-size parity sample: the first and the last `edge` coordinates
+    (the last quad's ragged tail included) and `n_windows` random windows of
+    `width` coordinates between them (about a million coordinates)."""
+    if d <= 2 * edge + width:
+        return windows(d)
+    rng = np.random.default_rng(seed)
+    blocks = (d - 2 * edge) // width
+    picks = np.sort(rng.choice(blocks, size=min(n_windows, blocks), replace=False))
+    return ([(0, edge)] + [(edge + int(b) * width, width) for b in picks] + [(d - edge, edge)])
+
+
 def sample_columns(d: int, head: int, tail: int, n_random: int, seed: int = 0):
     """Contiguous ranges (start, length) to compare: the first `head`
     coordinates, the last `tail` (ragged end of the last quad included) and
@@ -66,13 +85,22 @@ def sample_columns(d: int, head: int, tail: int, n_random: int, seed: int = 0):
     return ranges
 
 
+def oracle_ranges(w, ranges, steps: int, mode: int | None = None, c0: int = 0) -> list:
+    """oracle_range for every (start, length) window, run concurrently on the
+    host cores (one window per task; the oracle's ctypes calls release the
+    GIL and it keeps no shared state)."""
+    from concurrent.futures import ThreadPoolExecutor
+    threads = max(1, min(len(ranges), len(os.sched_getaffinity(0))))
+    with ThreadPoolExecutor(threads) as pool:
+        return list(pool.map(lambda r: oracle_range(w, c0 + r[0], r[1], steps, mode), ranges))
+
+
 def compare_ranges(run: rs.RelayRun, w, ranges, steps: int, mode: int | None = None, c0: int = 0):
     """Max parity error of x and of the last messages over the given ranges;
     asserts the counters are bit-exact."""
     gx, gm, ox, om = [], [], [], []
     counts = None
-    for start, length in ranges:
-        st = oracle_range(w, c0 + start, length, steps, mode)
+    for (start, length), st in zip(ranges, oracle_ranges(w, ranges, steps, mode, c0)):
         gx.append(run.x[:, start:start + length].double().cpu().numpy())
         gm.append(run.messages[:run.E, start:start + length].double().cpu().numpy())
         ox.append(st.x)

@@ -19,7 +19,8 @@ from oracle import oracle
 from paper_2110_04175_gb300 import build as rs_build
 from paper_2110_04175_gb300 import workloads as wl
 from tests import treeutil as tu
-from tests.gpu_util import RTOL, compare_ranges, gpu_run, oracle_range, parity_error, sample_columns
+from tests.gpu_util import (RTOL, c8_sample, compare_ranges, gpu_run, oracle_range, parity_error,
+                             windows)
 
 pytestmark = pytest.mark.gpu
 
@@ -226,11 +227,14 @@ FULL = [wl.binary16_resnet20(), wl.chain16_vgg11(), wl.binary32_bert()] + [
 
 @pytest.mark.parametrize("w", FULL, ids=lambda w: w.name)
 def test_full_size_workload_sampled(w):
-    """Full d and the workload's step count on the GPU; oracle on the first
-    2048 and last 1031 coordinates and 48 random ones."""
+    """Full d and the workload's step count on the GPU, in the launch
+    configuration bench.py times (stored centres, the automatic kernel
+    choice, the workload's rebuild rule).  The oracle checks every coordinate
+    of the ResNet-20-sized workload, and on the larger ones the first and
+    last 65,536 coordinates plus 1,024 random windows of 1,024."""
     _free()
-    run = gpu_run(w, w.steps)
-    ranges = sample_columns(w.d, 2048, 1031, 48, seed=w.n)
+    run = gpu_run(w, w.steps, objective="stored")
+    ranges = windows(w.d) if w.d < 1_000_000 else c8_sample(w.d, seed=w.n)
     ex, em = compare_ranges(run, w, ranges, w.steps)
     del run
     _free()
