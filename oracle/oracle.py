@@ -61,6 +61,9 @@ def _load():
         lib.oracle_normal.argtypes = [ctypes.c_uint64, ctypes.c_int64, ctypes.c_uint32,
                                       ctypes.c_uint32, ctypes.c_uint32]
         lib.oracle_normal.restype = ctypes.c_double
+        lib.oracle_fill_normals.argtypes = [ctypes.c_uint64, ctypes.c_int64, ctypes.c_int64,
+                                            ctypes.c_uint32, ctypes.c_uint32, ctypes.c_uint32, f64p]
+        lib.oracle_fill_normals.restype = ctypes.c_int
         lib.oracle_fill_mu.argtypes = [ctypes.c_int, ctypes.c_int, f64p, ctypes.c_double,
                                        ctypes.c_uint64, ctypes.c_int64, ctypes.c_int64, f64p]
         lib.oracle_fill_mu.restype = ctypes.c_int
@@ -130,8 +133,11 @@ def normal(seed: int, c: int, row: int, step: int, stream: int) -> float:
 
 
 def normals(seed: int, c0: int, length: int, row: int, step: int, stream: int) -> np.ndarray:
+    """oracle_normal for coordinates [c0, c0 + length) of (row, step, stream)."""
     lib = _load()
-    return np.array([lib.oracle_normal(seed, c0 + c, row, step, stream) for c in range(length)])
+    out = np.zeros(max(length, 0), dtype=np.float64)
+    _check(lib.oracle_fill_normals(seed, c0, length, row, step, stream, _ptr(out, ctypes.c_double)))
+    return out
 
 
 def _edges_arr(edges) -> np.ndarray:

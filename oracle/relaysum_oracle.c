@@ -218,6 +218,15 @@ int oracle_fill_mu(int n, int K, const double *mix, double mu_scale,
     return ORACLE_OK;
 }
 
+/* out[c] = oracle_normal(seed, c0 + c, row, step, stream) for c < len: the
+ * same numbers as one call per coordinate, for tests that need many. */
+int oracle_fill_normals(uint64_t seed, int64_t c0, int64_t len, uint32_t row, uint32_t step,
+                        uint32_t stream, double *out) {
+    if (len < 0 || c0 < 0 || (len > 0 && !out)) return ORACLE_EINVAL;
+    for (int64_t c = 0; c < len; ++c) out[c] = oracle_normal(seed, c0 + c, row, step, stream);
+    return ORACLE_OK;
+}
+
 /* x_i^0 = x0_std * N(c) for every worker i: one shared draw (stream 2),
  * because Alg. 1 starts all workers from the same model. */
 int oracle_fill_x0(int n, double x0_std, uint64_t seed, int64_t c0, int64_t len,

@@ -85,14 +85,19 @@ def sample_columns(d: int, head: int, tail: int, n_random: int, seed: int = 0):
     return ranges
 
 
-def oracle_ranges(w, ranges, steps: int, mode: int | None = None, c0: int = 0) -> list:
-    """oracle_range for every (start, length) window, run concurrently on the
-    host cores (one window per task; the oracle's ctypes calls release the
-    GIL and it keeps no shared state)."""
+def parallel_map(fn, items) -> list:
+    """fn over items on the host cores, in order: for oracle work, whose ctypes
+    calls release the GIL and which keeps no shared state."""
     from concurrent.futures import ThreadPoolExecutor
-    threads = max(1, min(len(ranges), len(os.sched_getaffinity(0))))
+    items = list(items)
+    threads = max(1, min(len(items), len(os.sched_getaffinity(0))))
     with ThreadPoolExecutor(threads) as pool:
-        return list(pool.map(lambda r: oracle_range(w, c0 + r[0], r[1], steps, mode), ranges))
+        return list(pool.map(fn, items))
+
+
+def oracle_ranges(w, ranges, steps: int, mode: int | None = None, c0: int = 0) -> list:
+    """oracle_range for every (start, length) window, run concurrently."""
+    return parallel_map(lambda r: oracle_range(w, c0 + r[0], r[1], steps, mode), ranges)
 
 
 def compare_ranges(run: rs.RelayRun, w, ranges, steps: int, mode: int | None = None, c0: int = 0):

@@ -11,7 +11,7 @@ import paper_2110_04175_gb300 as rs
 from oracle import oracle
 from paper_2110_04175_gb300 import build as rs_build
 from paper_2110_04175_gb300 import workloads as wl
-from tests.gpu_util import RTOL, parity_error, sample_columns
+from tests.gpu_util import RTOL, c8_sample, parallel_map, parity_error
 
 pytestmark = pytest.mark.gpu
 
@@ -46,29 +46,33 @@ def _run_both(w, steps, mode, optimizer=None, lost=None, ranges=None, objective=
         o = OPTS[optimizer]
         kw = dict(opt=o[0], beta1=o[1][1], beta2=o[1][2] if len(o[1]) > 2 else 0.0,
                   eps=o[1][3] if len(o[1]) > 3 else 0.0)
-    gx, gm, ox, om = [], [], [], []
-    counts = None
-    for start, length in ranges:
+    lr, sigma = float(np.float32(w.lr)), float(np.float32(w.sigma))
+
+    def oracle_window(r):
+        start, length = r
         st = oracle.State(w.n, w.edges, length, c0=start)
         st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
-        lr, sigma = float(np.float32(w.lr)), float(np.float32(w.sigma))
         if lost is None:
             st.advance(steps, lr, sigma, w.seed, mode, **kw)
         else:
             for t in range(steps):
                 st.advance(1, lr, sigma, w.seed, mode, drop=lost[t:t + 1], **kw)
+        return st
+
+    gx, gm, ox, om = [], [], [], []
+    counts = None
+    for (start, length), st in zip(ranges, parallel_map(oracle_window, ranges)):
         gx.append(run.x[:, start:start + length].double().cpu().numpy())
         gm.append(run.messages[:run.E, start:start + length].double().cpu().numpy())
         ox.append(st.x)
         om.append(st.msg)
         counts = st.counts
     assert np.array_equal(run.counts[:run.E].cpu().numpy(), counts)
-    ex = parity_error(np.concatenate(gx, 1), np.concatenate(ox, 1))
-    em = parity_error(np.concatenate(gm, 1), np.concatenate(om, 1))
+    gx, ox, gm, om = (np.concatenate(a, 1) for a in (gx, ox, gm, om))
     del run
     gc.collect()
     torch.cuda.empty_cache()
-    return ex, em
+    return parity_error(gx, ox), parity_error(gm, om)
 
 
 @pytest.mark.parametrize("objective", ["stored", "generated"])
@@ -84,14 +88,86 @@ def test_local_optimizers_every_coordinate(shape, n, d, optimizer, mode, objecti
     assert ex <= RTOL and em <= RTOL, (ex, em)
 
 
-@pytest.mark.parametrize("optimizer", ["nesterov", "adam"])
-def test_local_optimizers_full_size_sampled(optimizer):
-    """The 32-worker 1.1e8-parameter workload with each local optimiser (50
-    steps), oracle on the first/last coordinates and 32 random ones."""
+def test_nesterov_full_size_sampled():
+    """The 32-worker 1.1e8-parameter workload with Nesterov momentum (50
+    steps), oracle on the first and last 65,536 coordinates and 1,024 random
+    windows of 1,024."""
     w = wl.binary32_bert()
-    ranges = sample_columns(w.d, 1024, 1031, 32, seed=5)
-    ex, em = _run_both(w, w.steps, w.mode, optimizer, ranges=ranges)
+    ex, em = _run_both(w, w.steps, w.mode, "nesterov", ranges=c8_sample(w.d, seed=5))
     assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+def adam_rounding_bound(w, start, length, steps, beta1, beta2, eps):
+    """Per coordinate, how far fp32 rounding can move Adam's trajectory.
+
+    Adam's update divides by sqrt(v_hat) + eps, so a rounding error dg in a
+    gradient moves the update by about lr (1 - beta1) / (1 - beta1^k) dg /
+    (sqrt(v_hat) + eps): large wherever a worker's gradient is small
+    against its history.  The update's own rounding (a few ulp of |u|) adds
+    up too, since |u| stays near lr however small the gradient.  At the
+    first step the update is -lr g / (|g| + eps), in effect -lr sign(g):
+    within rounding of zero the sign itself is the decision, and the two
+    precisions may differ by 2 lr.  The relay and rebuild only average, so
+    per step the largest worker's error bounds the change at every worker.
+    dg is the fp32 rounding of the gradient's terms, 2^-23 (|x| + |mu| +
+    sigma |xi|), and the update's own rounding is taken as 8 ulp of |u|.
+    Returns (oracle state, amplified-gradient bound, own-rounding bound)."""
+    lr, sigma = float(np.float32(w.lr)), float(np.float32(w.sigma))
+    st = oracle.State(w.n, w.edges, length, c0=start)
+    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+    mu = st.mu.copy()
+    amplified = np.zeros(length)  # gradient rounding through 1 / (sqrt(v_hat) + eps), and flips
+    own = np.zeros(length)        # the update's own rounding
+    for t in range(steps):
+        x = st.x.copy()
+        xi = np.stack([oracle.normals(w.seed, start, length, row=i, step=t, stream=0) for i in range(w.n)])
+        g = (x - mu) + sigma * xi
+        dg = 2.0 ** -23 * (np.abs(x) + np.abs(mu) + sigma * np.abs(xi))
+        st.advance(1, lr, sigma, w.seed, w.mode, opt=oracle.OPT_ADAM, beta1=beta1, beta2=beta2, eps=eps)
+        vhat = st.s2 / (1.0 - beta2 ** (t + 1))
+        denom = np.sqrt(vhat) + eps
+        du = lr * (1.0 - beta1) / (1.0 - beta1 ** (t + 1)) * dg / denom
+        if t == 0:
+            du = np.where(np.abs(g) <= 4.0 * dg, 2.0 * lr, du)
+        amplified += du.max(axis=0)
+        # |u| stays near lr whatever |g| is
+        u = lr / (1.0 - beta1 ** (t + 1)) * np.abs(st.s1) / denom
+        own += (8.0 * 2.0 ** -24 * u).max(axis=0)
+    return st, amplified, own
+
+
+def test_adam_full_size_sampled():
+    """The 32-worker 1.1e8-parameter workload with Adam (50 steps), same
+    sample.  Every element meets 1e-5 of the parity metric plus 4x the
+    rounding bound of adam_rounding_bound (n times that for messages, sums
+    of up to n workers' values).  Fewer than 1 in 1,000 coordinates may
+    need more than the plain 1e-5 bar."""
+    w = wl.binary32_bert()
+    b1, b2, eps = OPTS["adam"][1][1:]
+    ranges = c8_sample(w.d, seed=5)
+    run = rs.RelayRun(w.n, w.d, w.edges, device="cuda:0", mode=w.mode, optimizer=OPTS["adam"][1])
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    for _ in range(w.steps):
+        run.step(w.lr, w.seed)
+    torch.cuda.synchronize()
+    res = parallel_map(lambda r: adam_rounding_bound(w, r[0], r[1], w.steps, b1, b2, eps), ranges)
+    gx = np.concatenate([run.x[:, s:s + l].double().cpu().numpy() for s, l in ranges], 1)
+    gm = np.concatenate([run.messages[:run.E, s:s + l].double().cpu().numpy() for s, l in ranges], 1)
+    assert np.array_equal(run.counts[:run.E].cpu().numpy(), res[0][0].counts)
+    del run
+    gc.collect()
+    torch.cuda.empty_cache()
+    ox = np.concatenate([r[0].x for r in res], 1)
+    om = np.concatenate([r[0].msg for r in res], 1)
+    amplified = np.concatenate([r[1] for r in res])
+    own = np.concatenate([r[2] for r in res])
+    for g, r, scale in ((gx, ox, 1.0), (gm, om, float(w.n))):
+        rms = float(np.sqrt(np.mean(r * r)))
+        plain = RTOL * np.maximum(np.abs(r), rms)
+        allowed = plain + 4.0 * scale * (amplified + own)[None, :]
+        assert np.all(np.abs(g - r) <= allowed), float(np.max(np.abs(g - r) - allowed))
+        # the allowance beyond the plain bar is needed on few coordinates
+        assert np.mean(np.any(np.abs(g - r) > plain, axis=0)) < 1e-3
 
 
 @pytest.mark.parametrize("mode", [0, 1])
@@ -115,7 +191,7 @@ def test_lost_messages_with_momentum_full_size_sampled():
     w = wl.Workload("binary16_d9231114", 16, wl.binary_tree(16), 9_231_114, wl.identity_mix(16),
                     1.0, 0.05, 0.05, 0.0, 60)
     lost = (np.random.default_rng(7).random((w.steps, w.E)) < 0.10).astype(np.uint8)
-    ranges = sample_columns(w.d, 1024, 1031, 32, seed=6)
+    ranges = c8_sample(w.d, seed=6)
     ex, em = _run_both(w, w.steps, 1, "nesterov", lost=lost, ranges=ranges)
     assert ex <= RTOL and em <= RTOL, (ex, em)
 
@@ -171,7 +247,8 @@ def test_other_algorithms_every_coordinate(shape, n, d, algorithm, lost_p):
 
 @pytest.mark.parametrize("algorithm", ["grad", "dme"])
 def test_other_algorithms_full_size_sampled(algorithm):
-    """The 64-worker torus spanning tree at d = 2.5e7, 100 steps."""
+    """The 64-worker torus spanning tree at d = 2.5e7, 100 steps; oracle on the
+    first and last 65,536 coordinates and 1,024 random windows of 1,024."""
     w = wl.sweep64("torus")
     run = rs.RelayRun(w.n, w.d, w.edges, device="cuda:0", algorithm=algorithm)
     run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
@@ -180,14 +257,19 @@ def test_other_algorithms_full_size_sampled(algorithm):
     for _ in range(w.steps):
         run.step(w.lr, w.seed)
     torch.cuda.synchronize()
-    gx, ox, gm, om = [], [], [], []
-    for start, length in sample_columns(w.d, 1024, 1031, 24, seed=8):
+    def oracle_window(r):
+        start, length = r
         st = oracle.State(w.n, w.edges, length, c0=start)
         st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
         if algorithm == "dme":
             st.x[:] = 0.0
         st.advance(w.steps, float(np.float32(w.lr)), float(np.float32(w.sigma)), w.seed, 1,
                    algo=ALGOS[algorithm])
+        return st
+
+    gx, ox, gm, om = [], [], [], []
+    ranges = c8_sample(w.d, seed=8)
+    for (start, length), st in zip(ranges, parallel_map(oracle_window, ranges)):
         gx.append(run.x[:, start:start + length].double().cpu().numpy())
         gm.append(run.messages[:run.E, start:start + length].double().cpu().numpy())
         ox.append(st.x)

@@ -56,6 +56,15 @@ def test_box_muller_outputs_are_standard_normal():
     assert abs(np.corrcoef(z[:, 0], z[:, 2])[0, 1]) < 0.05
 
 
+def test_vector_normals_equal_one_call_per_coordinate():
+    """oracle.normals (one C loop) returns exactly oracle_normal per coordinate."""
+    lib = oracle._load()
+    for seed, c0, row, step, stream in ((0, 0, 0, 0, 0), (99, 37, 5, 3, 0), (2**40 + 7, 1001, 31, 49, 1)):
+        got = oracle.normals(seed, c0, 67, row=row, step=step, stream=stream)
+        want = np.array([lib.oracle_normal(seed, c0 + c, row, step, stream) for c in range(67)])
+        assert np.array_equal(got, want)
+
+
 def test_streams_rows_steps_differ():
     base = oracle.normals(7, 0, 64, row=0, step=0, stream=0)
     for kw in (dict(row=1, step=0, stream=0), dict(row=0, step=1, stream=0),
