@@ -455,10 +455,13 @@ def run_native(args, w, rank: int, world: int):
 
 def run_graphed(args, w, run, dev, stream, rank: int, world: int):
     """Timed region = one replay of a CUDA graph holding the K steps (for
-    launch-bound small problems); the graph is captured after the warm-up."""
+    launch-bound small problems).  The graph is captured after the warm-up
+    and replayed once untimed first (the first launch of a graph also
+    uploads it); the timed replay runs the same K steps again."""
     import torch
     torch.cuda.synchronize(dev)
     g = run.capture(args.steps, w.lr, w.seed)
+    g.replay()
     torch.cuda.synchronize(dev)
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)

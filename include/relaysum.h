@@ -205,8 +205,12 @@ int relay_step_models(relay_handle *h, float *x, const float *msg_in, float *msg
                        relay_stream_t stream);
 
 /* One full RelaySGD iteration t: relay_step_counts, then
- * relay_step_models, enqueued back to back on `stream`.  The caller swaps
- * msg_in and msg_out before the next step (double-buffered messages). */
+ * relay_step_models, enqueued back to back on `stream`.  The step kernel is
+ * launched as a programmatic dependent of the counter kernel: it may be
+ * scheduled while the counter kernel runs and waits for it before reading
+ * the counters (relay_step_models called alone is an ordinary launch).  The
+ * caller swaps msg_in and msg_out before the next step (double-buffered
+ * messages). */
 int relay_step(relay_handle *h, float *x, const float *msg_in, float *msg_out,
                int32_t *counts, float lr, uint64_t seed, int64_t step,
                relay_stream_t stream);

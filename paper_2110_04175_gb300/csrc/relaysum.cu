@@ -178,6 +178,18 @@ __device__ __forceinline__ void st_stream(float* p, float4 v) {
     __stcs(reinterpret_cast<float4*>(p), v);
 }
 
+// ------------------------------------------------- programmatic dependent launch
+
+// relay_step launches the step kernel as a programmatic dependent of the
+// counter kernel: the counter kernel lets it be scheduled at once, and the
+// step kernel waits for the counter kernel's completion (and its writes)
+// before its first read of the counters.  Launched the ordinary way, the
+// wait returns immediately.
+__device__ __forceinline__ void allow_dependent_launch() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void wait_for_prior_grid() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ------------------------------------------------------------------ counters
 
 // c^t_{i->j} = 1 + sum_{k in N(i)\j} c^{t-1}_{k->i}: the incoming edge from
@@ -191,6 +203,7 @@ struct LostMask {
 
 __global__ void relay_counts_kernel(const __grid_constant__ Program prog, const __grid_constant__ LostMask lost,
                                     int has_lost, int32_t* counts, int64_t* dme_count) {
+    allow_dependent_launch();
     __shared__ int32_t c_old[kMaxE];
     const int E = prog.E;
     for (int e = threadIdx.x; e < E; e += blockDim.x) c_old[e] = counts[e];
@@ -422,6 +435,7 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
     __shared__ float s_scale[kMaxN];
     __shared__ float s_fill[kMaxN];
     const int n = prog.n;
+    wait_for_prior_grid();
     rebuild_factors(prog, a, s_scale, s_fill);
     __syncthreads();
     const Slots sl{slot_mem + threadIdx.x, static_cast<int>(blockDim.x)};
@@ -563,8 +577,6 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
     // regenerated centres are formed per row (the walk's cached centres are
     // the same normals mixed in the same order)
     constexpr int kObj = (OBJ == relaysum::kMuStored) ? relaysum::kMuStored : relaysum::kMuPerRow;
-    rebuild_factors(prog, a, s_scale, s_fill);
-    __syncthreads();
     const int i = static_cast<int>(threadIdx.x) / qb;
     const int qi = static_cast<int>(threadIdx.x) - i * qb;
     float4* const buf0 = node_mem + qi;                     // [e * qb]: m^t on edge e (even blocks)
@@ -583,6 +595,10 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
         xn = *reinterpret_cast<const float4*>(xrow + 4 * q);
         if (OBJ == relaysum::kMuStored) mn = ld_stream(murow + 4 * q);
     }
+    // x and mu are not written by the counter kernel; the counters are
+    wait_for_prior_grid();
+    rebuild_factors(prog, a, s_scale, s_fill);
+    __syncthreads();
     int parity = 0;
     for (int64_t b = blockIdx.x; b < nblk; b += gridDim.x, q += qstep, parity ^= 1) {
         float4* const m_new = parity ? buf1 : buf0;
@@ -766,6 +782,29 @@ int launch_status() {
     return cudaGetLastError() == cudaSuccess ? RELAY_OK : RELAY_ECUDA;
 }
 
+// Launches a step kernel; `after_counts` makes it a programmatic dependent of
+// the counter kernel just enqueued on the same stream (relay_step only).
+template <typename... Params, typename... Args>
+int launch_step_kernel(void (*kernel)(Params...), int grid, int threads, size_t smem, cudaStream_t stream,
+                       bool after_counts, Args... args) {
+    if (!after_counts) {
+        kernel<<<grid, threads, smem, stream>>>(args...);
+        return launch_status();
+    }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(static_cast<unsigned>(threads));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, kernel, args...) != cudaSuccess) return RELAY_ECUDA;
+    return launch_status();
+}
+
 // AUTO picks the node-parallel kernel below this many worker-quads (n times
 // the quads) when no worker has more than kRegDeg neighbours.  Measured on
 // one GB300 (whole step, L2 flushed, n = 8 to 64): the node kernel is ahead
@@ -783,7 +822,7 @@ int models_threads(int nslots) {
 }
 
 template <int OBJ, int OPT>
-int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
+int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream, bool after_counts) {
     int dev = 0;
     const int sms = device_sms(&dev);
     if (sms <= 0) return RELAY_ECUDA;
@@ -819,8 +858,8 @@ int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream
     const int64_t cap = static_cast<int64_t>(sms) * per_sm;
     const int grid = static_cast<int>(want < cap ? want : cap);
     const PhiloxKey mu_key = philox_key(static_cast<uint64_t>(h->obj.k0) | (static_cast<uint64_t>(h->obj.k1) << 32));
-    relay_models_kernel<OBJ, OPT><<<grid, threads, smem, stream>>>(h->prog, h->obj, mu_key, a);
-    return launch_status();
+    return launch_step_kernel(relay_models_kernel<OBJ, OPT>, grid, threads, smem, stream, after_counts, h->prog,
+                              h->obj, mu_key, a);
 }
 
 // Quads per CTA of the node-parallel kernel, threads = qb * n <= 1024: a
@@ -829,7 +868,7 @@ int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream
 int nodes_qb(int n) { return n <= 16 ? 32 : n <= 64 ? 16 : n <= 128 ? 8 : 4; }
 
 template <int OBJ, int OPT>
-int launch_nodes(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
+int launch_nodes(const relay_handle* h, const ModelArgs& a, cudaStream_t stream, bool after_counts) {
     int dev = 0;
     const int sms = device_sms(&dev);
     if (sms <= 0) return RELAY_ECUDA;
@@ -864,8 +903,8 @@ int launch_nodes(const relay_handle* h, const ModelArgs& a, cudaStream_t stream)
     const int64_t cap = static_cast<int64_t>(sms) * per_sm;
     const int grid = static_cast<int>(want < cap ? want : cap);
     const PhiloxKey mu_key = philox_key(static_cast<uint64_t>(h->obj.k0) | (static_cast<uint64_t>(h->obj.k1) << 32));
-    relay_nodes_kernel<OBJ, OPT><<<grid, threads, smem, stream>>>(h->prog, h->obj, mu_key, a, qb);
-    return launch_status();
+    return launch_step_kernel(relay_nodes_kernel<OBJ, OPT>, grid, threads, smem, stream, after_counts, h->prog,
+                              h->obj, mu_key, a, qb);
 }
 
 // AUTO: the walk keeps every array's traffic at one pass with one thread
@@ -881,15 +920,16 @@ bool use_nodes(const relay_handle* h) {
 }
 
 template <int OPT>
-int launch_models_obj(const relay_handle* h, const ModelArgs& a, cudaStream_t stream) {
+int launch_models_obj(const relay_handle* h, const ModelArgs& a, cudaStream_t stream, bool after_counts) {
     if (use_nodes(h)) {
-        if (h->obj.source == relaysum::kMuStored) return launch_nodes<relaysum::kMuStored, OPT>(h, a, stream);
-        return launch_nodes<relaysum::kMuPerRow, OPT>(h, a, stream);
+        if (h->obj.source == relaysum::kMuStored)
+            return launch_nodes<relaysum::kMuStored, OPT>(h, a, stream, after_counts);
+        return launch_nodes<relaysum::kMuPerRow, OPT>(h, a, stream, after_counts);
     }
     switch (h->obj.source) {
-        case relaysum::kMuStored: return launch_models<relaysum::kMuStored, OPT>(h, a, stream);
-        case relaysum::kMuPerRow: return launch_models<relaysum::kMuPerRow, OPT>(h, a, stream);
-        default: return launch_models<relaysum::kMuCachedCentres, OPT>(h, a, stream);
+        case relaysum::kMuStored: return launch_models<relaysum::kMuStored, OPT>(h, a, stream, after_counts);
+        case relaysum::kMuPerRow: return launch_models<relaysum::kMuPerRow, OPT>(h, a, stream, after_counts);
+        default: return launch_models<relaysum::kMuCachedCentres, OPT>(h, a, stream, after_counts);
     }
 }
 
@@ -1138,9 +1178,11 @@ int relay_step_counts(relay_handle* h, int32_t* counts, relay_stream_t stream) {
     return launch_status();
 }
 
-int relay_step_models(relay_handle* h, float* x, const float* msg_in, float* msg_out,
-                      const int32_t* counts, float lr, uint64_t seed, int64_t step,
-                      relay_stream_t stream) {
+// The step kernel's launch; `after_counts`: relay_step's counter kernel was
+// just enqueued on `stream`, so the step may start as its programmatic
+// dependent.
+static int step_models(relay_handle* h, float* x, const float* msg_in, float* msg_out, const int32_t* counts,
+                       float lr, uint64_t seed, int64_t step, relay_stream_t stream, bool after_counts) {
     const int rc = check_step_args(h, x, msg_in, msg_out, counts, lr, step);
     if (rc != RELAY_OK) return rc;
     if (h->d == 0) return RELAY_OK;
@@ -1175,10 +1217,16 @@ int relay_step_models(relay_handle* h, float* x, const float* msg_in, float* msg
         a.adam_ibc2 = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(static_cast<double>(h->beta2), k)));
     }
     switch (h->opt) {
-        case 0: return launch_models_obj<0>(h, a, stream);
-        case 1: return launch_models_obj<1>(h, a, stream);
-        default: return launch_models_obj<2>(h, a, stream);
+        case 0: return launch_models_obj<0>(h, a, stream, after_counts);
+        case 1: return launch_models_obj<1>(h, a, stream, after_counts);
+        default: return launch_models_obj<2>(h, a, stream, after_counts);
     }
+}
+
+int relay_step_models(relay_handle* h, float* x, const float* msg_in, float* msg_out,
+                      const int32_t* counts, float lr, uint64_t seed, int64_t step,
+                      relay_stream_t stream) {
+    return step_models(h, x, msg_in, msg_out, counts, lr, seed, step, stream, false);
 }
 
 int relay_step(relay_handle* h, float* x, const float* msg_in, float* msg_out, int32_t* counts, float lr,
@@ -1187,9 +1235,11 @@ int relay_step(relay_handle* h, float* x, const float* msg_in, float* msg_out, i
     // rejected step leaves the counters untouched
     int rc = check_step_args(h, x, msg_in, msg_out, counts, lr, step);
     if (rc != RELAY_OK) return rc;
+    // relay_step_counts launches only when there are counters to update
+    const bool counted = h->prog.E > 0 || h->algo == RELAY_ALGO_DME;
     rc = relay_step_counts(h, counts, stream);
     if (rc != RELAY_OK) return rc;
-    return relay_step_models(h, x, msg_in, msg_out, counts, lr, seed, step, stream);
+    return step_models(h, x, msg_in, msg_out, counts, lr, seed, step, stream, counted);
 }
 
 int relay_nbar(const relay_handle* h, const int32_t* counts_host, int32_t* nbar_host) {
