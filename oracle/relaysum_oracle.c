@@ -41,7 +41,14 @@
  * (0, 1) into the normals of coordinates 4q, 4q+1 (cos, sin) and words (2, 3)
  * into those of 4q+2, 4q+3.
  *
- * parity pinned: see tests/test_oracle_pins.py and tests/test_bruteforce.py.
+ * parity pinned: every function here is checked against something other than
+ * itself -- published Philox known-answer vectors, closed forms (counters,
+ * subtree sums, fixed points, plain SGD and all-reduce special cases), an
+ * exact-rational routing brute force on every tree of up to 6 nodes, the
+ * paper's stacked-delay matrix form, torch.optim's SGD/Adam, and brute-force
+ * restatements of Algorithms 5 and 6: tests/test_oracle_pins.py,
+ * tests/test_bruteforce.py, tests/test_matrix_form.py and
+ * tests/test_oracle_extensions.py.
  */
 #define _USE_MATH_DEFINES
 #include <math.h>
