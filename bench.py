@@ -358,6 +358,7 @@ def run_native(args, w, rank: int, world: int):
                    else "relay_models_kernel")
 
     def one_step(ev=None):
+        torch.cuda.nvtx.range_push(f"relay_step {run.t}")  # a named range per step for profilers
         for k, tr in enumerate(run.trees):
             if args.lost_prob > 0:  # messages lost in transit this step (Section 4.4)
                 rs.relay_set_lost_messages(tr.h, lost_rng.random(tr.E) < args.lost_prob)
@@ -372,6 +373,7 @@ def run_native(args, w, rank: int, world: int):
                 ev[k][2].record(stream)
             tr.cur = 1 - tr.cur
         run.t += 1
+        torch.cuda.nvtx.range_pop()
 
     T = len(run.trees)
     for _ in range(args.warmup):
