@@ -223,8 +223,10 @@ int relay_nbar(const relay_handle *h, const int32_t *counts_host, int32_t *nbar_
  * number of shared-memory accumulator slots per thread, the visit order
  * (int32 [n]), per node 10 ints {deg, pos_base, parent_pos, recv_slot,
  * acc_slot, parent_acc, fin_parent, parent, tot_slot, flags} (int32 [n][10];
- * flags bit 0: recv_slot holds the parent's total) and per position 3 ints
- * {in_edge, out_edge, slot} (int32 [E][3]); any output pointer may be NULL. */
+ * flags bit 0: recv_slot holds the parent's total) and per position 4 ints
+ * {in_edge, out_edge, slot, rebuild_in_edge} (int32 [E][4]; the last lists
+ * each worker's incoming edges in the order its rebuild adds them); any
+ * output pointer may be NULL. */
 int relay_program(const relay_handle *h, int32_t *nslots, int32_t *order, int32_t *node_rec,
                   int32_t *pos_rec);
 

@@ -286,12 +286,12 @@ def relay_nbar(h, counts_host) -> np.ndarray:
 
 
 def relay_program(h):
-    """(nslots, order[n], node_rec[n][10], pos_rec[E][3]) of the fused kernel's visit program."""
+    """(nslots, order[n], node_rec[n][10], pos_rec[E][4]) of the step kernels' visit program."""
     n, E = h.n, relay_num_edges(h)
     nslots = ctypes.c_int32()
     order = np.zeros(n, dtype=np.int32)
     node = np.zeros((n, 10), dtype=np.int32)
-    pos = np.zeros((max(E, 1), 3), dtype=np.int32)
+    pos = np.zeros((max(E, 1), 4), dtype=np.int32)
     _check(_load().relay_program(_h(h), ctypes.addressof(nslots), order.ctypes.data,
                                  node.ctypes.data, pos.ctypes.data), "relay_program")
     return int(nslots.value), order, node, pos[:E]

@@ -1269,9 +1269,10 @@ int relay_program(const relay_handle* h, int32_t* nslots, int32_t* order, int32_
     }
     if (pos_rec)
         for (int e = 0; e < p.E; ++e) {
-            pos_rec[3 * e] = p.pos_in[e];
-            pos_rec[3 * e + 1] = p.pos_out[e];
-            pos_rec[3 * e + 2] = p.pos_slot[e];
+            pos_rec[4 * e] = p.pos_in[e];
+            pos_rec[4 * e + 1] = p.pos_out[e];
+            pos_rec[4 * e + 2] = p.pos_slot[e];
+            pos_rec[4 * e + 3] = p.rb_in[e];
         }
     return RELAY_OK;
 }

@@ -179,6 +179,56 @@ def test_program_with_lost_messages_matches_oracle(shape, mode):
     check_tree(n, edges, mode, steps=6, L=2, p_lost=0.25)
 
 
+def _rebuild_orders(h, n):
+    """Per worker: the incoming edges in the order the walk adds them (its
+    DFS parent's at its own visit, then each child's at that child's visit),
+    derived from the visit order and the parents alone; and the program's
+    rebuild-order table, which the node-parallel kernel follows."""
+    _, order, node, pos = rs.relay_program(h)
+    src, dst = rs.relay_edges(h)
+    edge = {(int(a), int(b)): e for e, (a, b) in enumerate(zip(src, dst))}
+    walk = {i: [] for i in range(n)}
+    for i in order:
+        par = node[i][7]
+        if par >= 0:
+            walk[i].append(edge[(int(par), int(i))])   # the parent's message, at i's visit
+            walk[par].append(edge[(int(i), int(par))])  # i's message joins the parent's sum
+    table = {i: [int(pos[node[i][1] + k][3]) for k in range(node[i][0])] for i in range(n)}
+    return walk, table
+
+
+def _trees_for_orders():
+    out = [(n, e) for n in range(1, 7) for e in tu.all_trees(n)]
+    out += [(64, wl.star(64)), (64, wl.torus_spanning_tree(8, 8, 0)), (40, wl.random_tree(40, 1)),
+            (32, wl.binary_tree(32)), (16, wl.double_binary_trees(16)[1]), (256, wl.chain(256))]
+    return out
+
+
+def test_rebuild_order_table_follows_the_walk():
+    """For every tree up to 6 nodes and the workload trees, the table lists
+    each worker's incoming edges exactly once, in the walk's order; adding
+    float32 messages in that order reproduces the walk's sums bit for bit."""
+    rng = np.random.default_rng(3)
+    for n, edges in _trees_for_orders():
+        edges = np.asarray(edges, np.int32).reshape(-1, 2)
+        h = rs.relay_create(n, 4, edges)
+        walk, table = _rebuild_orders(h, n)
+        src, dst = rs.relay_edges(h)
+        E = 2 * (n - 1)
+        m = rng.normal(size=(E, 8)).astype(np.float32)
+        base = rng.normal(size=(n, 8)).astype(np.float32)
+        for i in range(n):
+            assert table[i] == walk[i], (n, i, table[i], walk[i])
+            assert sorted(table[i]) == sorted(e for e in range(E) if dst[e] == i)
+            a = base[i].copy()
+            b = base[i].copy()
+            for e in walk[i]:
+                a = a + m[e]
+            for e in table[i]:
+                b = b + m[e]
+            assert np.array_equal(a, b)
+
+
 def test_slot_counts_of_workload_trees():
     """The walk keeps the shared-memory footprint small: O(1) on chains,
     O(depth) on balanced trees, the hub degree on a star."""
