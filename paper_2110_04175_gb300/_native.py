@@ -336,7 +336,9 @@ class RelayRun:
         kernel: "auto", "walk" or "nodes" (relay_set_kernel)."""
         import torch
         if objective not in ("stored", "generated"):
-            raise ValueError(objective)
+            raise ValueError(f"objective must be 'stored' or 'generated', not {objective!r}")
+        if kernel not in ("auto", "walk", "nodes"):
+            raise ValueError(f"kernel must be 'auto', 'walk' or 'nodes', not {kernel!r}")
         trees = list(edges) if isinstance(edges, (list, tuple)) else [edges]
         self.objective = objective
         self.n, self.d, self.c0 = n, d, c0

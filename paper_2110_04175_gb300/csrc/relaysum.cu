@@ -584,7 +584,7 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
     float4* const m_old = node_mem + 2 * prog.E * qb + qi;  // [e * qb]: m^{t-1} (wide nodes)
     const NodeRec r = prog.node[i];
     const float* const xrow = a.x + i * a.ld_x;
-    const float* const murow = a.mu + i * a.ld_x;  // read only for a stored mu
+    const float* const murow = (OBJ == relaysum::kMuStored) ? a.mu + i * a.ld_x : nullptr;
     const int64_t nblk = (a.nquads + qb - 1) / qb;
     const int64_t qstep = static_cast<int64_t>(gridDim.x) * qb;
     // x (and a stored mu) of this thread's next block are loaded one block
