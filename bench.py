@@ -427,7 +427,7 @@ def run_native(args, w, rank: int, world: int):
     achieved = alg_bytes / (mean_models_ms / 1e3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4),
-                "traffic": traffic_per_launch(w, args.objective, kernel_name),
+                "traffic": traffic_per_launch(w, args.objective, kernel_name, args.optimizer),
                 "kernel": kernel_name, "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "algorithmic_bytes_rule": "4 d (2n + 2E) [+ 4 d n x optimiser-state rows]",
@@ -596,18 +596,18 @@ def run_e2e(args, w, run, dev, stream, world: int):
             "copy_frac": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9 / link["both_gbs"], 3)}
 
 
-def traffic_per_launch(w, objective: str, kernel: str = "relay_models_kernel"):
+def traffic_per_launch(w, objective: str, kernel: str = "relay_models_kernel", optimizer: str = "sgd"):
     """DRAM bytes per launch of the step kernel from the committed ncu
-    summary for this kernel, workload and objective source
-    (profiles/traffic.txt), or None when no capture of the current kernel
-    exists for it."""
+    summary for this kernel, workload, objective source and local optimiser
+    (profiles/traffic.txt; plain entries are SGD), or None when no capture of
+    the current kernel exists for it."""
+    key = f"{kernel}/{w.name}/{objective}" + ("" if optimizer == "sgd" else f"/{optimizer}")
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     try:
         with open(path) as f:
             for line in f:
                 parts = line.split()
-                if len(parts) == 2 and not line.startswith("#") and \
-                        parts[0] == f"{kernel}/{w.name}/{objective}":
+                if len(parts) == 2 and not line.startswith("#") and parts[0] == key:
                     return int(parts[1])
     except OSError:
         pass
