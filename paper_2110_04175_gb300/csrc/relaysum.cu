@@ -821,6 +821,29 @@ int models_threads(int nslots) {
     return t;
 }
 
+// Opts `Kernel` in to the full dynamic shared memory once per device and
+// returns its resident CTAs per SM for (threads, smem).  Both are cached per
+// device (queried once, not per step: steps may be captured into CUDA
+// graphs); each kernel instantiation has its own cache.  0 on a CUDA error.
+template <auto Kernel>
+int resident_ctas(int dev, int threads, size_t smem) {
+    static std::atomic<bool> smem_set[kMaxDevices];
+    if (dev >= kMaxDevices || !smem_set[dev].load()) {
+        if (cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) != cudaSuccess)
+            return 0;
+        if (dev < kMaxDevices) smem_set[dev].store(true);
+    }
+    static std::atomic<int64_t> occ_cache[kMaxDevices];
+    const int64_t key = static_cast<int64_t>(smem) * 1024 + threads;
+    const int64_t cached = dev < kMaxDevices ? occ_cache[dev].load() : 0;
+    if (cached != 0 && (cached >> 8) == key) return static_cast<int>(cached & 0xFF);
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, Kernel, threads, smem) != cudaSuccess || per_sm <= 0)
+        return 0;
+    if (dev < kMaxDevices) occ_cache[dev].store((key << 8) | (per_sm & 0xFF));
+    return per_sm;
+}
+
 template <int OBJ, int OPT>
 int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream, bool after_counts) {
     int dev = 0;
@@ -830,30 +853,8 @@ int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream
     const int threads = models_threads(per_thread);
     const size_t smem = static_cast<size_t>(per_thread) * threads * 16;
     if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
-    // opt in to the full shared memory once per device (the 48 KB default
-    // covers dynamic AND static shared memory)
-    static std::atomic<bool> smem_set[kMaxDevices];
-    if ((dev >= kMaxDevices || !smem_set[dev].load())) {
-        if (cudaFuncSetAttribute(relay_models_kernel<OBJ, OPT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kMaxSmem) != cudaSuccess)
-            return RELAY_ECUDA;
-        if (dev < kMaxDevices) smem_set[dev].store(true);
-    }
-    // resident CTAs per SM, cached per device for the last shared-memory size
-    // (queried once, not per step: steps may be captured into CUDA graphs)
-    static std::atomic<int64_t> occ_cache[kMaxDevices];
-    int per_sm = 0;
-    const int64_t key = static_cast<int64_t>(smem) * 1024 + threads;
-    const int64_t cached = dev < kMaxDevices ? occ_cache[dev].load() : 0;
-    if (cached != 0 && (cached >> 8) == key) {
-        per_sm = static_cast<int>(cached & 0xFF);
-    } else {
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_models_kernel<OBJ, OPT>, threads,
-                                                          smem) != cudaSuccess ||
-            per_sm <= 0)
-            return RELAY_ECUDA;
-        if (dev < kMaxDevices) occ_cache[dev].store((key << 8) | (per_sm & 0xFF));
-    }
+    const int per_sm = resident_ctas<relay_models_kernel<OBJ, OPT>>(dev, threads, smem);
+    if (per_sm <= 0) return RELAY_ECUDA;
     const int64_t want = (a.nquads + threads - 1) / threads;
     const int64_t cap = static_cast<int64_t>(sms) * per_sm;
     const int grid = static_cast<int>(want < cap ? want : cap);
@@ -878,27 +879,8 @@ int launch_nodes(const relay_handle* h, const ModelArgs& a, cudaStream_t stream,
     for (int i = 0; i < h->prog.n; ++i) wide = wide || h->prog.node[i].deg > kRegDeg;
     const size_t smem = static_cast<size_t>(wide ? 3 : 2) * h->prog.E * qb * 16;
     if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
-    static std::atomic<bool> smem_set[kMaxDevices];
-    if ((dev >= kMaxDevices || !smem_set[dev].load())) {
-        if (cudaFuncSetAttribute(relay_nodes_kernel<OBJ, OPT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kMaxSmem) != cudaSuccess)
-            return RELAY_ECUDA;
-        if (dev < kMaxDevices) smem_set[dev].store(true);
-    }
-    // resident CTAs per SM, cached per device (threads and smem depend on n only)
-    static std::atomic<int64_t> occ_cache[kMaxDevices];
-    int per_sm = 0;
-    const int64_t key = static_cast<int64_t>(smem) * 1024 + threads;
-    const int64_t cached = dev < kMaxDevices ? occ_cache[dev].load() : 0;
-    if (cached != 0 && (cached >> 8) == key) {
-        per_sm = static_cast<int>(cached & 0xFF);
-    } else {
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, relay_nodes_kernel<OBJ, OPT>, threads,
-                                                          smem) != cudaSuccess ||
-            per_sm <= 0)
-            return RELAY_ECUDA;
-        if (dev < kMaxDevices) occ_cache[dev].store((key << 8) | (per_sm & 0xFF));
-    }
+    const int per_sm = resident_ctas<relay_nodes_kernel<OBJ, OPT>>(dev, threads, smem);
+    if (per_sm <= 0) return RELAY_ECUDA;
     const int64_t want = (a.nquads + qb - 1) / qb;
     const int64_t cap = static_cast<int64_t>(sms) * per_sm;
     const int grid = static_cast<int>(want < cap ? want : cap);
