@@ -219,6 +219,39 @@ def test_streams_are_respected():
     assert torch.equal(run.x, ref.x)
 
 
+@pytest.mark.parametrize("shape,n,d,kernel,algorithm", [
+    ("chain", 8, 4096, "nodes", "relaysgd"), ("binary", 16, 65537, "walk", "relaysgd"),
+    ("star", 9, 1031, "walk", "relaysgd"), ("binary", 15, 2053, "nodes", "dme"),
+    ("single", 1, 517, "auto", "relaysgd"), ("single", 1, 517, "auto", "dme")])
+def test_overlapped_step_launch_equals_separate_launches(shape, n, d, kernel, algorithm):
+    """relay_step starts the step kernel as a programmatic dependent of the
+    counter kernel; that changes only scheduling, so 60 such steps must equal
+    60 steps of relay_step_counts and relay_step_models launched apart, bit
+    for bit (including n = 1, where no counter kernel runs unless mean
+    estimation needs its counts)."""
+    edges = {"chain": wl.chain(n), "binary": wl.binary_tree(n), "star": wl.star(n),
+             "single": np.zeros((0, 2), np.int32)}[shape]
+    runs = []
+    for _ in range(2):
+        run = rs.RelayRun(n, d, edges, device="cuda:0", kernel=kernel, algorithm=algorithm)
+        run.init(0.1, 5, wl.identity_mix(n), 1.0, 6, 0.1)
+        runs.append(run)
+    a, b = runs
+    for t in range(60):
+        a.step(0.05, 5)
+        tr = b.trees[0]
+        rs.relay_step_counts(tr.h, tr.counts)
+        rs.relay_step_models(tr.h, b.x, tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, 0.05, 5, t)
+        tr.cur = 1 - tr.cur
+    torch.cuda.synchronize()
+    assert torch.equal(a.x[:, :d], b.x[:, :d])
+    if a.E:
+        assert torch.equal(a.messages[:a.E, :d], b.trees[0].messages[:a.E, :d])
+        assert torch.equal(a.counts[:a.E], b.trees[0].counts[:a.E])
+    if algorithm == "dme":
+        assert torch.equal(a.trees[0].dme_count, b.trees[0].dme_count)
+
+
 # -------------------------------------------------- full-size workloads
 
 FULL = [wl.binary16_resnet20(), wl.chain16_vgg11(), wl.binary32_bert()] + [
