@@ -116,3 +116,32 @@ def compare_ranges(run: rs.RelayRun, w, ranges, steps: int, mode: int | None = N
     ex = parity_error(np.concatenate(gx, axis=1), np.concatenate(ox, axis=1))
     em = parity_error(np.concatenate(gm, axis=1), np.concatenate(om, axis=1)) if run.E else 0.0
     return ex, em
+
+
+def adam_step_bound(x, mu, xi, sigma: float, m, v, lr: float, beta1: float, beta2: float, eps: float,
+                    t: int) -> np.ndarray:
+    """Per coordinate, how far fp32 rounding can move one Adam step (t from
+    0) of any worker, from the oracle's state before the step (x, mu, the
+    noise xi) and after it (first and second moments m, v), all [n][len].
+
+    Adam divides by sqrt(v_hat) + eps, so a rounding error dg in a gradient
+    moves the update by lr (1 - beta1) / (1 - beta1^k) dg / (sqrt(v_hat) +
+    eps): large wherever a worker's gradient is small against its history.
+    The update's own rounding (8 ulp of |u|) adds up too, since |u| stays
+    near lr however small the gradient.  At the first step the update is
+    -lr g / (|g| + eps), in effect -lr sign(g) when eps is tiny: within
+    rounding of zero the sign is a decision that two precisions may take
+    differently, a difference of 2 lr.  dg is the fp32 rounding of the
+    gradient's terms, 2^-23 (|x| + |mu| + sigma |xi|).  The relay and
+    rebuild only average, so the largest worker's value bounds the step's
+    effect on every worker; summed over steps it bounds the trajectory."""
+    g = (x - mu) + sigma * xi
+    dg = 2.0 ** -23 * (np.abs(x) + np.abs(mu) + sigma * np.abs(xi))
+    k = t + 1
+    denom = np.sqrt(v / (1.0 - beta2 ** k)) + eps
+    du = lr * (1.0 - beta1) / (1.0 - beta1 ** k) * dg / denom
+    if t == 0:
+        du = np.where(np.abs(g) <= 4.0 * dg, 2.0 * lr, du)
+    du = du + 8.0 * 2.0 ** -24 * (lr / (1.0 - beta1 ** k) * np.abs(m) / denom)
+    return du.max(axis=0)
+
