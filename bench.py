@@ -590,7 +590,8 @@ def run_e2e(args, w, run, dev, stream, world: int):
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
             "path": "HostRelayRun: state in pinned host memory, streamed through the GPU in "
                     f"{host.nchunks} chunks of {cw} coordinates ({args.copy_streams} copy-in / "
-                    f"kernel / {args.copy_streams} copy-out streams), copies inside the timed region",
+                    f"kernel / {args.copy_streams} copy-out streams), copies inside the timed region; "
+                    "x, the counters and the message rows a later step reads cross the link",
             "copy_gbs": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9, 1),
             "host_link": link,
             "copy_frac": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9 / link["both_gbs"], 3)}

@@ -10,10 +10,15 @@ one contiguous block).  A step:
 2. streams the chunks through a ring of device buffers on three CUDA
    streams -- host-to-device copies, the fused kernel (relay_step_models on
    a handle whose coordinate offset is the chunk's absolute position), and
-   device-to-host copies -- so both copy directions and the kernels overlap
-   (message rows arriving at a leaf are never read by the kernel and are not
-   copied in);
+   device-to-host copies -- so both copy directions and the kernels overlap;
 3. copies the counters out.
+
+Only the message rows that a later step reads cross the link.  A message
+arriving at a leaf is consumed by the leaf's rebuild in the step that forms
+it (a leaf's only outgoing message excludes its only incoming one), so those
+rows are neither copied in nor copied out: the host keeps x, the counters
+and every message row the next step reads, and messages() marks the rows it
+does not keep as NaN.
 
 Ordering: every reuse of a device buffer waits for the copy-out of the chunk
 that last used it; a chunk's copy-in waits for the previous step's copy-out
@@ -58,22 +63,20 @@ class HostRelayRun:
         h0 = self.handles[self.widths[0]]
         self.E = nat.relay_num_edges(h0)
         E1 = max(self.E, 1)
-        # message rows the kernel reads: all but those arriving at a leaf (a
-        # leaf's only outgoing message excludes its only incoming one), as
-        # contiguous runs; the others are not copied in (their device rows
-        # are never read)
+        # message rows a later step reads: all but those arriving at a leaf,
+        # as contiguous runs; only these cross the link, in both directions
         if self.E > 0:
             _, _, node, pos = nat.relay_program(h0)
             unread = {int(pos[node[i][1]][0]) for i in range(n) if node[i][0] == 1}
-            rows = [e for e in range(self.E) if e not in unread]
+            self.kept_rows = [e for e in range(self.E) if e not in unread]
         else:
-            rows = []
-        self.read_runs = []
-        for e in rows:
-            if self.read_runs and self.read_runs[-1][1] == e:
-                self.read_runs[-1][1] = e + 1
+            self.kept_rows = []
+        self.kept_runs = []
+        for e in self.kept_rows:
+            if self.kept_runs and self.kept_runs[-1][1] == e:
+                self.kept_runs[-1][1] = e + 1
             else:
-                self.read_runs.append([e, e + 1])
+                self.kept_runs.append([e, e + 1])
         pin = dict(dtype=torch.float32, pin_memory=True)
         self.x_h = torch.empty(self.nchunks, n, self.cw, **pin)
         self.msg_h = [torch.empty(self.nchunks, E1, self.cw, **pin) for _ in range(2)]
@@ -141,7 +144,7 @@ class HostRelayRun:
                 s_in.wait_event(self.out_done[b])
                 s_in.wait_event(self.out_done_k[k])
                 self.xb[b].copy_(self.x_h[k], non_blocking=True)
-                for lo, hi in self.read_runs:
+                for lo, hi in self.kept_runs:
                     self.mib[b][lo:hi].copy_(src[k][lo:hi], non_blocking=True)
                 self.in_done[b].record(s_in)
             self.s_comp.wait_event(self.in_done[b])
@@ -151,7 +154,8 @@ class HostRelayRun:
             with torch.cuda.stream(s_out):
                 s_out.wait_event(self.comp_done[b])
                 self.x_h[k].copy_(self.xb[b], non_blocking=True)
-                dst[k].copy_(self.mob[b], non_blocking=True)
+                for lo, hi in self.kept_runs:
+                    dst[k][lo:hi].copy_(self.mob[b][lo:hi], non_blocking=True)
                 self.out_done[b].record(s_out)
                 self.out_done_k[k].record(s_out)
         with torch.cuda.stream(self.s_out):
@@ -167,16 +171,21 @@ class HostRelayRun:
 
     def bytes_per_step(self):
         """(host-to-device, device-to-host) bytes copied per step."""
-        rows_in = sum(hi - lo for lo, hi in self.read_runs)
-        h2d = (self.x_h.numel() + self.nchunks * rows_in * self.cw + self.counts_h.numel()) * 4
-        d2h = (self.x_h.numel() + self.msg_h[0].numel() + self.counts_h.numel()) * 4
-        return h2d, d2h
+        rows = len(self.kept_rows)
+        per_direction = (self.x_h.numel() + self.nchunks * rows * self.cw + self.counts_h.numel()) * 4
+        return per_direction, per_direction
 
     def models(self):
         """x as a host [n][d] array (a copy)."""
         return self.x_h.permute(1, 0, 2).reshape(self.n, -1)[:, :self.d].clone()
 
     def messages(self):
-        """m^{t-1} as a host [E][d] array (a copy)."""
+        """m^{t-1} as a host [E][d] array (a copy); rows the host does not keep
+        (messages arriving at leaves, which no later step reads) are NaN."""
+        import torch
         m = self.msg_h[self.cur]
-        return m.permute(1, 0, 2).reshape(m.shape[1], -1)[:self.E, :self.d].clone()
+        out = m.permute(1, 0, 2).reshape(m.shape[1], -1)[:self.E, :self.d].clone()
+        dropped = [e for e in range(self.E) if e not in set(self.kept_rows)]
+        if dropped:
+            out[dropped] = torch.nan
+        return out

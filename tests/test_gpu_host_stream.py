@@ -1,4 +1,6 @@
-"""The host-state streaming mode equals the fully resident run, bit for bit."""
+"""The host-state streaming mode equals the fully resident run, bit for bit,
+on everything it keeps: the models, the counters and every message row that
+a later step reads (all but the rows arriving at leaves)."""
 import numpy as np
 import pytest
 import torch
@@ -20,9 +22,11 @@ def _gpu():
     ("binary", 16, 1_000_003, 1 << 18, 3),   # 4 chunks, ragged last one
     ("star", 12, 70_001, 1 << 14, 2),        # wide node, 5 chunks, 2 buffers
     ("chain", 5, 1_000, 1 << 12, 3),         # a single chunk
+    ("pair", 2, 5_000, 1 << 12, 2),          # two leaves: no message row is kept
 ])
 def test_host_stream_equals_resident_run(shape, n, d, chunk, buffers):
-    edges = {"binary": wl.binary_tree(n), "star": wl.star(n), "chain": wl.chain(n)}[shape]
+    edges = {"binary": wl.binary_tree(n), "star": wl.star(n), "chain": wl.chain(n),
+             "pair": wl.chain(n)}[shape]
     w = wl.Workload(shape, n, edges, d, wl.identity_mix(n), 1.0, 0.05, 0.05, 0.1, 7)
     dev = rs.RelayRun(n, d, edges, device="cuda:0")
     dev.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
@@ -34,5 +38,13 @@ def test_host_stream_equals_resident_run(shape, n, d, chunk, buffers):
     host.sync()
     torch.cuda.synchronize()
     assert torch.equal(host.models(), dev.x[:, :d].cpu())
-    assert torch.equal(host.messages(), dev.messages[:dev.E, :d].cpu())
     assert torch.equal(host.counts_h[:dev.E], dev.counts[:dev.E].cpu())
+    # the kept rows are exactly those whose receiver is not a leaf
+    src, dst = rs.relay_edges(dev.h)
+    degree = np.bincount(np.asarray(dst), minlength=n)
+    assert host.kept_rows == [e for e in range(dev.E) if degree[dst[e]] > 1]
+    got = host.messages()
+    kept = host.kept_rows
+    assert torch.equal(got[kept], dev.messages[:dev.E, :d].cpu()[kept])
+    dropped = [e for e in range(dev.E) if e not in kept]
+    assert torch.isnan(got[dropped]).all()
