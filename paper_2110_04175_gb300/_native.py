@@ -489,8 +489,37 @@ class RelayRun:
         relay_set_lost_messages(self.trees[tree].h, lost)
 
     def step(self, lr: float, seed: int, stream=None):
-        for tr in self.trees:
+        """Enqueues one step on `stream` (default: the current stream).  With
+        several trees (double binary trees) the windows, which share no
+        data, run on streams forked from `stream` and joined back to it, so
+        one window's last wave overlaps the next window's start."""
+        if len(self.trees) == 1:
+            tr = self.trees[0]
             relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed,
                        self.t, stream)
             tr.cur = 1 - tr.cur
+            self.t += 1
+            return
+        import torch
+        if stream is None:
+            main = torch.cuda.current_stream(self.device)
+        elif isinstance(stream, int):
+            main = torch.cuda.ExternalStream(stream) if stream else torch.cuda.default_stream(self.device)
+        else:
+            main = stream
+        if getattr(self, "_side", None) is None:
+            self._side = [torch.cuda.Stream(self.device) for _ in self.trees]
+        fork = torch.cuda.Event()
+        fork.record(main)
+        joins = []
+        for tr, side in zip(self.trees, self._side):
+            side.wait_event(fork)
+            relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed,
+                       self.t, side)
+            tr.cur = 1 - tr.cur
+            done = torch.cuda.Event()
+            done.record(side)
+            joins.append(done)
+        for done in joins:
+            main.wait_event(done)
         self.t += 1
