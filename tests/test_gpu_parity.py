@@ -19,8 +19,8 @@ from oracle import oracle
 from paper_2110_04175_gb300 import build as rs_build
 from paper_2110_04175_gb300 import workloads as wl
 from tests import treeutil as tu
-from tests.gpu_util import (RTOL, c8_sample, compare_ranges, gpu_run, oracle_range, parity_error,
-                             windows)
+from tests.gpu_util import (RTOL, c8_sample, compare_ranges, gpu_run, oracle_range, parallel_map,
+                             parity_error, windows)
 
 pytestmark = pytest.mark.gpu
 
@@ -272,6 +272,36 @@ def test_full_size_workload_sampled(w):
     del run
     _free()
     assert ex <= RTOL and em <= RTOL, (ex, em)
+
+
+def test_double16_full_size_sampled():
+    """Double binary trees (Section 3) at the VGG-11 size, 200 steps, as
+    bench.py runs them (stored centres, the two windows on forked streams).
+    In each tree's coordinate window the oracle runs that tree on the first
+    and last 65,536 coordinates and 1,024 random windows of 1,024."""
+    _free()
+    w = wl.double16_vgg11()
+    run = gpu_run(w, w.steps, objective="stored")
+    lr, sigma = float(np.float32(w.lr)), float(np.float32(w.sigma))
+    for tr, edges in zip(run.trees, w.edges):
+        ranges = [(tr.col0 + s, l) for s, l in c8_sample(tr.d, seed=tr.col0 + 1)]
+
+        def oracle_window(r, edges=edges):
+            st = oracle.State(w.n, edges, r[1], c0=r[0])
+            st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+            st.advance(w.steps, lr, sigma, w.seed, w.mode)
+            return st
+
+        states = parallel_map(oracle_window, ranges)
+        gx = np.concatenate([run.x[:, s:s + l].double().cpu().numpy() for s, l in ranges], 1)
+        gm = np.concatenate([tr.messages[:tr.E, s - tr.col0:s - tr.col0 + l].double().cpu().numpy()
+                             for s, l in ranges], 1)
+        ox = np.concatenate([st.x for st in states], 1)
+        om = np.concatenate([st.msg for st in states], 1)
+        assert np.array_equal(tr.counts[:tr.E].cpu().numpy(), states[0].counts)
+        assert parity_error(gx, ox) <= RTOL and parity_error(gm, om) <= RTOL
+    del run
+    _free()
 
 
 def test_binary16_resnet20_every_coordinate_mode0():
