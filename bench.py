@@ -426,6 +426,8 @@ def run_native(args, w, rank: int, world: int):
     total_ms = reduce_max(total_ms, world)
     steps_per_s = world * args.steps / (total_ms / 1e3)
 
+    # several steps per call, on the resident run (before run_e2e frees it)
+    fused = run_fused(args, w, run, dev, stream, world) if args.fused_steps > 0 else None
     # end to end: state in pinned host memory, copied in and out every step
     e2e = None
     if args.e2e_steps > 0:
@@ -470,8 +472,54 @@ def run_native(args, w, rank: int, world: int):
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": workload_config(w, world, args, dev), "roofline": roofline, "cpu_baseline": cpu,
             "e2e": e2e, "gpu_launches": 2 * T * args.steps, "clocks": clocks.summary(),
-            "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1)}
+            "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1),
+            "fused_steps": fused}
     print(json.dumps(line), flush=True)
+
+
+def run_fused(args, w, run, dev, stream, world: int) -> dict:
+    """The same workload through relay_steps: K steps per call, the state
+    kept on chip between them (the result equals K relay_step calls bit for
+    bit).  Its HBM traffic is one read and one write of the state per call,
+    so its rate is not an HBM roofline figure: the per-step line above is.
+    Calls are repeated for about half a second after one untimed call."""
+    import torch
+
+    import paper_2110_04175_gb300 as rs
+
+    if not run.trees:
+        raise RuntimeError("run_fused needs the resident run (run_e2e frees it)")
+    K = args.fused_steps
+    run.steps(K, w.lr, w.seed, stream)
+    torch.cuda.synchronize(dev)
+    probe = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    probe[0].record(stream)
+    run.steps(K, w.lr, w.seed, stream)
+    probe[1].record(stream)
+    torch.cuda.synchronize(dev)
+    calls = max(1, min(1000, int(500.0 / max(probe[0].elapsed_time(probe[1]), 1e-3))))
+    calls = int(reduce_max(float(calls), world))  # the same count on every rank
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    ev[0].record(stream)
+    for _ in range(calls):
+        run.steps(K, w.lr, w.seed, stream)
+    ev[1].record(stream)
+    torch.cuda.synchronize(dev)
+    ms = reduce_max(ev[0].elapsed_time(ev[1]), world)
+    fused = all(rs.relay_get_steps_kernel(tr.h) == rs.RELAY_KERNEL_FUSED for tr in run.trees)
+    E, state_rows = w.E, {"sgd": 0, "nesterov": 1, "adam": 2}[args.optimizer]
+    mu_rows = w.n if args.objective == "stored" else 0
+    # per call: read x, mu, the state, m^{t0-1}; write x, the state and the last two steps' messages
+    per_call = 4 * w.d * (w.n + mu_rows + state_rows * w.n + E + w.n + state_rows * w.n + min(K, 2) * E)
+    launches = (-(-K // 64)) * (1 + (E > 0 or args.algorithm == "dme")) if fused else 2 * K
+    return {"value": round(world * K * calls / (ms / 1e3), 4), "unit": "steps/s", "steps_per_call": K,
+            "calls": calls, "ms_per_step": round(ms / (K * calls), 5),
+            "kernel": "relay_fused_steps_kernel" if fused else "one relay_step per step (a wide node)",
+            "launches_per_call": launches * len(run.trees),
+            "hbm_bytes_per_call": per_call if fused else None,
+            "note": "several steps per launch, the state on chip between them; not an HBM roofline figure"}
 
 
 def run_graphed(args, w, run, dev, stream, rank: int, world: int):
@@ -660,6 +708,9 @@ def main(argv=None):
                    help="probability that each message is lost in transit, per step")
     p.add_argument("--objective", choices=["generated", "stored"], default="stored",
                    help="regenerate the centres mu in the kernel, or read a stored mu array")
+    p.add_argument("--fused-steps", type=int, default=64,
+                   help="also time relay_steps with this many steps per call (0: skip); reported "
+                        "under 'fused_steps', beside the per-step headline")
     p.add_argument("--d", type=int, default=None,
                    help="override the workload's d (small cases for profiling; not a bench line)")
     args = p.parse_args(argv)

@@ -215,6 +215,34 @@ int relay_step(relay_handle *h, float *x, const float *msg_in, float *msg_out,
                int32_t *counts, float lr, uint64_t seed, int64_t step,
                relay_stream_t stream);
 
+/* k consecutive iterations t0, t0+1, ..., t0+k-1 of Algorithm 1 (k >= 0),
+ * equal bit for bit to k relay_step calls that alternate the two message
+ * buffers: iteration t0+j reads msg_a if j is even (msg_b if odd) and writes
+ * the other.  On entry msg_a holds m^{t0-1}; on return the buffer written
+ * last holds m^{t0+k-1} (msg_b if k is odd, msg_a if even), the other one
+ * m^{t0+k-2} (k >= 2), counts hold c^{t0+k-1}, and x, the optimiser state
+ * and the mean-estimation counts have advanced k steps.  The lost-message
+ * mask in force applies to every one of the k steps.  Every coordinate
+ * evolves on its own, so the steps run without a round trip through HBM:
+ * each CTA keeps its quads' models and optimiser state in registers and
+ * their messages in shared memory for up to 64 steps per launch (then a
+ * 1-CTA launch advances the counters).  That fused kernel is taken under
+ * RELAY_KERNEL_NODES, and under RELAY_KERNEL_AUTO when no worker has more
+ * than 4 neighbours; otherwise (RELAY_KERNEL_WALK, or a wide node such as a
+ * star's hub, whose threads would hold their CTA at every step) relay_steps
+ * enqueues k relay_step calls.  Arguments and errors as relay_step
+ * (x, msg_a, msg_b, counts, lr, seed; t0 the noise counter of the first
+ * step), plus RELAY_EINVAL when k < 0 or t0 + k > 2^32.  The buffers are
+ * caller-owned device memory; nothing is allocated. */
+int relay_steps(relay_handle *h, float *x, float *msg_a, float *msg_b, int32_t *counts,
+                float lr, uint64_t seed, int64_t t0, int64_t k, relay_stream_t stream);
+
+/* The path relay_steps takes on this handle: RELAY_KERNEL_FUSED (several
+ * steps per launch), else the per-step kernel of relay_get_kernel; or
+ * RELAY_EINVAL. */
+#define RELAY_KERNEL_FUSED 3
+int relay_get_steps_kernel(const relay_handle *h);
+
 /* nbar_i = 1 + sum of the counters arriving at i, from host counters
  * (int32 [E]) into nbar_host (int32 [n]).  Host arithmetic only. */
 int relay_nbar(const relay_handle *h, const int32_t *counts_host, int32_t *nbar_host);

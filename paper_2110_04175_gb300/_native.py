@@ -25,6 +25,7 @@ RELAY_ALGO_DME = 2
 RELAY_KERNEL_AUTO = 0
 RELAY_KERNEL_WALK = 1
 RELAY_KERNEL_NODES = 2
+RELAY_KERNEL_FUSED = 3
 
 _lock = threading.Lock()
 _lib = None
@@ -55,6 +56,7 @@ def _load():
             "relay_set_rebuild_mode": (ctypes.c_int, [vp, i32]),
             "relay_set_kernel": (ctypes.c_int, [vp, i32]),
             "relay_get_kernel": (ctypes.c_int, [vp]),
+            "relay_get_steps_kernel": (ctypes.c_int, [vp]),
             "relay_set_strides": (ctypes.c_int, [vp, i64, i64]),
             "relay_set_local_optimizer": (ctypes.c_int, [vp, i32, f32, f32, f32, vp, vp]),
             "relay_set_lost_messages": (ctypes.c_int, [vp, vp]),
@@ -67,6 +69,7 @@ def _load():
             "relay_step_counts": (ctypes.c_int, [vp, vp, vp]),
             "relay_step_models": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, vp]),
             "relay_step": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, vp]),
+            "relay_steps": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, i64, vp]),
             "relay_nbar": (ctypes.c_int, [vp, vp, vp]),
             "relay_program": (ctypes.c_int, [vp, vp, vp, vp, vp]),
             "relay_metrics_workspace": (i64, [vp]),
@@ -192,6 +195,14 @@ def relay_get_kernel(h) -> int:
     return k
 
 
+def relay_get_steps_kernel(h) -> int:
+    """RELAY_KERNEL_FUSED when relay_steps runs several steps per launch, else
+    the per-step kernel it repeats."""
+    k = _load().relay_get_steps_kernel(_h(h))
+    _check(min(k, 0), "relay_get_steps_kernel")
+    return k
+
+
 def relay_set_strides(h, ld_x: int, ld_msg: int):
     _check(_load().relay_set_strides(_h(h), int(ld_x), int(ld_msg)), "relay_set_strides")
 
@@ -256,6 +267,13 @@ def relay_step_models(h, x, msg_in, msg_out, counts, lr: float, seed: int, step:
 def relay_step(h, x, msg_in, msg_out, counts, lr: float, seed: int, step: int, stream=None):
     _check(_load().relay_step(_h(h), _ptr(x), _ptr(msg_in), _ptr(msg_out), _ptr(counts),
                               float(lr), int(seed), int(step), _stream(stream)), "relay_step")
+
+
+def relay_steps(h, x, msg_a, msg_b, counts, lr: float, seed: int, t0: int, k: int, stream=None):
+    """k steps t0 .. t0+k-1 in one launch per 64 steps; msg_a holds m^{t0-1}, and the
+    result equals k relay_step calls alternating msg_a and msg_b, bit for bit."""
+    _check(_load().relay_steps(_h(h), _ptr(x), _ptr(msg_a), _ptr(msg_b), _ptr(counts),
+                               float(lr), int(seed), int(t0), int(k), _stream(stream)), "relay_steps")
 
 
 def relay_metrics_workspace(h) -> int:
@@ -488,17 +506,14 @@ class RelayRun:
         """Messages of the next steps lost in transit on tree `tree` (E flags or None)."""
         relay_set_lost_messages(self.trees[tree].h, lost)
 
-    def step(self, lr: float, seed: int, stream=None):
-        """Enqueues one step on `stream` (default: the current stream).  With
-        several trees (double binary trees) the windows, which share no
-        data, run on streams forked from `stream` and joined back to it, so
-        one window's last wave overlaps the next window's start."""
+    def _per_tree(self, issue, stream):
+        """Calls issue(tree, stream) for every tree.  One tree runs on
+        `stream` (default: the current stream).  With several trees (double
+        binary trees) the windows, which share no data, run on streams forked
+        from `stream` and joined back to it, so one window's last wave
+        overlaps the next window's start."""
         if len(self.trees) == 1:
-            tr = self.trees[0]
-            relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed,
-                       self.t, stream)
-            tr.cur = 1 - tr.cur
-            self.t += 1
+            issue(self.trees[0], stream)
             return
         import torch
         if stream is None:
@@ -514,12 +529,30 @@ class RelayRun:
         joins = []
         for tr, side in zip(self.trees, self._side):
             side.wait_event(fork)
-            relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed,
-                       self.t, side)
-            tr.cur = 1 - tr.cur
+            issue(tr, side)
             done = torch.cuda.Event()
             done.record(side)
             joins.append(done)
         for done in joins:
             main.wait_event(done)
+
+    def step(self, lr: float, seed: int, stream=None):
+        """Enqueues one step (relay_step per tree) on `stream`."""
+        def issue(tr, s):
+            relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed, self.t, s)
+            tr.cur = 1 - tr.cur
+
+        self._per_tree(issue, stream)
         self.t += 1
+
+    def steps(self, k: int, lr: float, seed: int, stream=None):
+        """Enqueues k steps with relay_steps (the models and messages stay on
+        chip between them): the same state, bit for bit, as k step() calls."""
+        k = int(k)
+
+        def issue(tr, s):
+            relay_steps(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed, self.t, k, s)
+            tr.cur ^= k & 1
+
+        self._per_tree(issue, stream)
+        self.t += k

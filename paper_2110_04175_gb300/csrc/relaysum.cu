@@ -201,6 +201,18 @@ struct LostMask {
     __host__ __device__ __forceinline__ bool operator()(int e) const { return (w[e >> 5] >> (e & 31)) & 1u; }
 };
 
+// c^t of directed edge e from c^{t-1}; a lost message carries no count.
+__device__ __forceinline__ int32_t next_count(const Program& prog, const LostMask& lost, int has_lost,
+                                              const int32_t* c_old, int e) {
+    const NodeRec r = prog.node[prog.edge_src[e]];
+    int32_t s = 1;
+    for (int p = 0; p < r.deg; ++p) {
+        const int in = prog.pos_in[r.pos_base + p];
+        if (in != (e ^ 1)) s += c_old[in];
+    }
+    return (has_lost && lost(e)) ? 0 : s;
+}
+
 __global__ void relay_counts_kernel(const __grid_constant__ Program prog, const __grid_constant__ LostMask lost,
                                     int has_lost, int32_t* counts, int64_t* dme_count) {
     allow_dependent_launch();
@@ -208,15 +220,7 @@ __global__ void relay_counts_kernel(const __grid_constant__ Program prog, const 
     const int E = prog.E;
     for (int e = threadIdx.x; e < E; e += blockDim.x) c_old[e] = counts[e];
     __syncthreads();
-    for (int e = threadIdx.x; e < E; e += blockDim.x) {
-        const NodeRec r = prog.node[prog.edge_src[e]];
-        int32_t s = 1;
-        for (int p = 0; p < r.deg; ++p) {
-            const int in = prog.pos_in[r.pos_base + p];
-            if (in != (e ^ 1)) s += c_old[in];
-        }
-        counts[e] = (has_lost && lost(e)) ? 0 : s;  // a lost message carries no count
-    }
+    for (int e = threadIdx.x; e < E; e += blockDim.x) counts[e] = next_count(prog, lost, has_lost, c_old, e);
     if (dme_count) {  // Alg. 5: s_i += 1 + sum_j c^t_{j->i}
         __syncthreads();
         for (int i = threadIdx.x; i < prog.n; i += blockDim.x) {
@@ -226,6 +230,33 @@ __global__ void relay_counts_kernel(const __grid_constant__ Program prog, const 
             dme_count[i] += nb;
         }
     }
+}
+
+// The counters (and the mean-estimation counts) advanced by k steps, for
+// relay_steps: one CTA of blockDim >= n threads, the counters of the two
+// step parities in shared memory, one barrier per step.
+__global__ void relay_counts_steps_kernel(const __grid_constant__ Program prog,
+                                          const __grid_constant__ LostMask lost, int has_lost, int32_t* counts,
+                                          int64_t* dme_count, int k) {
+    __shared__ int32_t c[2][kMaxE];
+    const int E = prog.E;
+    for (int e = threadIdx.x; e < E; e += blockDim.x) c[1][e] = counts[e];
+    __syncthreads();
+    int64_t received = 0;  // worker threadIdx.x: sum over the k steps of 1 + sum_j c^t_{j->i}
+    for (int j = 0; j < k; ++j) {
+        const int32_t* c_old = c[(j + 1) & 1];
+        int32_t* c_new = c[j & 1];
+        for (int e = threadIdx.x; e < E; e += blockDim.x) c_new[e] = next_count(prog, lost, has_lost, c_old, e);
+        __syncthreads();
+        if (dme_count && threadIdx.x < prog.n) {
+            const NodeRec r = prog.node[threadIdx.x];
+            int64_t nb = 1;
+            for (int p = 0; p < r.deg; ++p) nb += c_new[prog.pos_in[r.pos_base + p]];
+            received += nb;
+        }
+    }
+    for (int e = threadIdx.x; e < E; e += blockDim.x) counts[e] = c[(k - 1) & 1][e];
+    if (dme_count && threadIdx.x < prog.n) dme_count[threadIdx.x] += received;
 }
 
 // --------------------------------------------------------------- fused step
@@ -341,29 +372,40 @@ __device__ __noinline__ void visit_wide(const Program& prog, const NodeRec& r, c
 //   Nesterov: m = beta1 m + g;  u = -lr (g + beta1 m)          (state s1 = m)
 //   Adam:     m = beta1 m + (1 - beta1) g;  v = beta2 v + (1 - beta2) g^2;
 //             u = -adam_step m / (sqrt(v) adam_ibc2 + eps)     (s1 = m, s2 = v)
+// The rule on the optimiser state (m, v) held in registers; adam_step and
+// adam_ibc2 are the factors of this step.
 template <int OPT>
-__device__ __forceinline__ float4 local_update(const ModelArgs& a, int i, int64_t q, float4 g) {
+__device__ __forceinline__ float4 update_rule(const ModelArgs& a, float adam_step, float adam_ibc2, float4 g,
+                                              float4& m, float4& v) {
     if (OPT == 0) return scale4(g, -a.lr);
-    float4* pm = reinterpret_cast<float4*>(a.s1 + i * a.ld_x + 4 * q);
-    float4 m = *pm;
     if (OPT == 1) {
         m = make_float4(fmaf(a.beta1, m.x, g.x), fmaf(a.beta1, m.y, g.y), fmaf(a.beta1, m.z, g.z),
                         fmaf(a.beta1, m.w, g.w));
-        __stcs(pm, m);
         return make_float4(-a.lr * fmaf(a.beta1, m.x, g.x), -a.lr * fmaf(a.beta1, m.y, g.y),
                            -a.lr * fmaf(a.beta1, m.z, g.z), -a.lr * fmaf(a.beta1, m.w, g.w));
     }
-    float4* pv = reinterpret_cast<float4*>(a.s2 + i * a.ld_x + 4 * q);
-    float4 v = *pv;
     const float c1 = 1.0f - a.beta1, c2 = 1.0f - a.beta2;
     m = make_float4(fmaf(a.beta1, m.x, c1 * g.x), fmaf(a.beta1, m.y, c1 * g.y), fmaf(a.beta1, m.z, c1 * g.z),
                     fmaf(a.beta1, m.w, c1 * g.w));
     v = make_float4(fmaf(a.beta2, v.x, c2 * g.x * g.x), fmaf(a.beta2, v.y, c2 * g.y * g.y),
                     fmaf(a.beta2, v.z, c2 * g.z * g.z), fmaf(a.beta2, v.w, c2 * g.w * g.w));
-    __stcs(pm, m);
-    __stcs(pv, v);
-    auto upd = [&](float mm, float vv) { return -a.adam_step * mm / fmaf(sqrtf(vv), a.adam_ibc2, a.eps); };
+    auto upd = [&](float mm, float vv) { return -adam_step * mm / fmaf(sqrtf(vv), adam_ibc2, a.eps); };
     return make_float4(upd(m.x, v.x), upd(m.y, v.y), upd(m.z, v.z), upd(m.w, v.w));
+}
+
+// One step's update with the state read from and written back to HBM.
+template <int OPT>
+__device__ __forceinline__ float4 local_update(const ModelArgs& a, int i, int64_t q, float4 g) {
+    float4 m = make_float4(0.f, 0.f, 0.f, 0.f), v = m;
+    if (OPT == 0) return update_rule<OPT>(a, a.adam_step, a.adam_ibc2, g, m, v);
+    float4* pm = reinterpret_cast<float4*>(a.s1 + i * a.ld_x + 4 * q);
+    float4* pv = reinterpret_cast<float4*>(a.s2 + i * a.ld_x + 4 * q);
+    m = *pm;
+    if (OPT == 2) v = *pv;
+    const float4 u = update_rule<OPT>(a, a.adam_step, a.adam_ibc2, g, m, v);
+    __stcs(pm, m);
+    if (OPT == 2) __stcs(pv, v);
+    return u;
 }
 
 // mu_i for quad q: read, or regenerated exactly as relay_fill_mu_kernel
@@ -387,6 +429,22 @@ __device__ __forceinline__ float4 centre(const Objective& obj, const PhiloxKey& 
 // with acc = fill * x + x^{t+1/2} + incoming messages.
 //   mode 0: x' = acc / nbar (Alg. 1).  mode 1: x' = (acc + (n - nbar) x) / n
 //   (robust rule), the fill term folded into the accumulator up front.
+__device__ __forceinline__ void worker_factors(const ModelArgs& a, int n, int nbar, float& scale, float& fill) {
+    if (a.algo == 1) {  // x' = x + (u + sum m) / n
+        scale = 1.0f / static_cast<float>(n);
+        fill = static_cast<float>(n);
+    } else if (a.algo == 2) {  // y' = y + dhat + sum m
+        scale = 1.0f;
+        fill = 1.0f;
+    } else if (a.mode == 0) {
+        scale = 1.0f / static_cast<float>(nbar);
+        fill = 0.0f;
+    } else {
+        scale = 1.0f / static_cast<float>(n);
+        fill = static_cast<float>(n - nbar);
+    }
+}
+
 __device__ __forceinline__ void rebuild_factors(const Program& prog, const ModelArgs& a, float* s_scale,
                                                 float* s_fill) {
     const int n = prog.n;
@@ -394,35 +452,30 @@ __device__ __forceinline__ void rebuild_factors(const Program& prog, const Model
         const NodeRec r = prog.node[i];
         int nbar = 1;
         for (int p = 0; p < r.deg; ++p) nbar += __ldg(a.counts + prog.pos_in[r.pos_base + p]);
-        if (a.algo == 1) {  // x' = x + (u + sum m) / n
-            s_scale[i] = 1.0f / static_cast<float>(n);
-            s_fill[i] = static_cast<float>(n);
-        } else if (a.algo == 2) {  // y' = y + dhat + sum m
-            s_scale[i] = 1.0f;
-            s_fill[i] = 1.0f;
-        } else if (a.mode == 0) {
-            s_scale[i] = 1.0f / static_cast<float>(nbar);
-            s_fill[i] = 0.0f;
-        } else {
-            s_scale[i] = 1.0f / static_cast<float>(n);
-            s_fill[i] = static_cast<float>(n - nbar);
-        }
+        worker_factors(a, n, nbar, s_scale[i], s_fill[i]);
     }
 }
 
 // The relayed value of worker i at quad q: x^{t+1/2} = x + u (Alg. 1), the
 // update u (Alg. 6) or the sample mu + sigma xi (Alg. 5), with
 // g = (x - mu) + sigma xi and z the worker's noise normals.
-template <int OPT>
-__device__ __forceinline__ float4 relayed_value(const ModelArgs& a, int i, int64_t q, float4 xv, float4 mv,
-                                                float4 z) {
+// `update` maps g to u (and advances the optimiser state).
+template <typename Update>
+__device__ __forceinline__ float4 relayed_with(const ModelArgs& a, float4 xv, float4 mv, float4 z,
+                                               Update update) {
     if (a.algo == 2)
         return make_float4(fmaf(a.sigma, z.x, mv.x), fmaf(a.sigma, z.y, mv.y), fmaf(a.sigma, z.z, mv.z),
                            fmaf(a.sigma, z.w, mv.w));
     const float4 g = make_float4(fmaf(a.sigma, z.x, xv.x - mv.x), fmaf(a.sigma, z.y, xv.y - mv.y),
                                  fmaf(a.sigma, z.z, xv.z - mv.z), fmaf(a.sigma, z.w, xv.w - mv.w));
-    const float4 u = local_update<OPT>(a, i, q, g);
+    const float4 u = update(g);
     return (a.algo == 1) ? u : add4(xv, u);
+}
+
+template <int OPT>
+__device__ __forceinline__ float4 relayed_value(const ModelArgs& a, int i, int64_t q, float4 xv, float4 mv,
+                                                float4 z) {
+    return relayed_with(a, xv, mv, z, [&](float4 g) { return local_update<OPT>(a, i, q, g); });
 }
 
 // OBJ: where mu comes from (ObjectiveSource).  OPT: the local optimiser
@@ -633,6 +686,164 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
     }
 }
 
+// ------------------------------------------------ several steps per launch
+
+// relay_steps: k consecutive steps in one launch, in the node-parallel
+// layout.  Every coordinate evolves on its own (the counters are the same
+// for all of them), so a CTA carries its qb quads of every worker through
+// all k steps without hearing from another CTA: models, centres and
+// optimiser state stay in registers, the messages of the step just taken
+// in shared memory, and the CTA advances its own copy of the counters.  HBM
+// is read once (x, mu, the optimiser state, m^{t0-1}) and written once (x,
+// the state, and the messages of the last two steps, which k relay_step
+// calls leave in the two buffers).  Each step is the node kernel's
+// arithmetic in the node kernel's order, so the result equals k relay_step
+// calls bit for bit.
+constexpr int kMaxFusedSteps = 64;  // steps per launch (Adam's per-step factors ride in the parameters)
+
+struct FusedSteps {
+    int32_t k;                        // steps in this launch, 1 .. kMaxFusedSteps
+    float* msg[2];                    // step t0 + j reads msg[j & 1] and writes msg[(j + 1) & 1]
+    float adam_step[kMaxFusedSteps];  // Adam's factors of step t0 + j
+    float adam_ibc2[kMaxFusedSteps];
+};
+
+// Outgoing messages of worker i from its incoming ones in shared memory
+// (`prev`, this thread's column), with node_small's / node_wide's arithmetic.
+// They go to `cur`, and to HBM at `out` (row e at out + e * ld_m) unless null.
+template <int D>
+__device__ __forceinline__ void fused_small(const Program& prog, const NodeRec& r, const ModelArgs& a, float4 xh,
+                                            const float4* prev, float4* cur, int qb, float* out) {
+    float4 m[D];
+#pragma unroll
+    for (int s = 0; s < D; ++s) m[s] = prev[prog.pos_in[r.pos_base + s] * qb];
+    float4 pre[D];
+    pre[0] = xh;
+#pragma unroll
+    for (int s = 1; s < D; ++s) pre[s] = add4(pre[s - 1], m[s - 1]);
+    float4 suf[D];
+    suf[D - 1] = m[D - 1];
+#pragma unroll
+    for (int s = D - 2; s >= 0; --s) suf[s] = add4(m[s], suf[s + 1]);
+#pragma unroll
+    for (int s = 0; s < D; ++s) {
+        const int e = prog.pos_out[r.pos_base + s];
+        const float4 o = delivered(a, e, (s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]));
+        cur[e * qb] = o;
+        if (out) st_stream(out + e * a.ld_m, o);
+    }
+}
+
+__device__ __noinline__ void fused_wide(const Program& prog, const NodeRec& r, const ModelArgs& a, float4 xh,
+                                        const float4* prev, float4* cur, int qb, float* out) {
+    const int D = r.deg;
+    const int base = r.pos_base;
+    float4 total = xh;
+    for (int s = D - 1; s >= 0; --s) total = add4(total, prev[prog.pos_in[base + s] * qb]);
+    for (int s = 0; s < D; ++s) {
+        const int e = prog.pos_out[base + s];
+        const float4 o = delivered(a, e, sub4(total, prev[prog.pos_in[base + s] * qb]));
+        cur[e * qb] = o;
+        if (out) st_stream(out + e * a.ld_m, o);
+    }
+}
+
+// blockDim.x = qb * n <= 1024, threads worker-major as in relay_nodes_kernel.
+// Dynamic shared memory: two [E][qb] float4 message buffers, buffer j & 1
+// holding the messages of step t0 + j (buffer 1 starts with m^{t0-1}), then
+// the rebuild factors (scale, fill) of every worker and step, [k][n] float2.
+// The counters, hence the factors, are the same for every quad: the CTA
+// advances them through the k steps once, before its first quads.  One
+// barrier per step: a thread can write a buffer again only two steps later,
+// after every thread has passed the barrier between, i.e. finished reading it.
+template <int OBJ, int OPT>
+__global__ void __launch_bounds__(1024)
+relay_fused_steps_kernel(const __grid_constant__ Program prog, const __grid_constant__ Objective obj,
+                         const __grid_constant__ PhiloxKey mu_key, const __grid_constant__ ModelArgs a,
+                         const __grid_constant__ FusedSteps fs, int qb) {
+    extern __shared__ float4 fused_mem[];
+    __shared__ int32_t c_mem[2][kMaxE];  // counters of the step parities
+    constexpr int kObj = (OBJ == relaysum::kMuStored) ? relaysum::kMuStored : relaysum::kMuPerRow;
+    const int tid = static_cast<int>(threadIdx.x);
+    const int i = tid / qb;
+    const int qi = tid - i * qb;
+    const int n = prog.n;
+    const int E = prog.E;
+    const NodeRec r = prog.node[i];
+    const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+    float2* const factors = reinterpret_cast<float2*>(fused_mem + 2 * E * qb);  // [j * n + i]
+    for (int e = tid; e < E; e += blockDim.x) c_mem[1][e] = a.counts[e];  // c^{t0-1}
+    __syncthreads();
+    for (int j = 0; j < fs.k; ++j) {
+        const int32_t* const c_old = c_mem[(j + 1) & 1];
+        int32_t* const c_new = c_mem[j & 1];
+        for (int e = tid; e < E; e += blockDim.x) c_new[e] = next_count(prog, a.lost, a.has_lost, c_old, e);
+        __syncthreads();
+        for (int w = tid; w < n; w += blockDim.x) {
+            const NodeRec rw = prog.node[w];
+            int nbar = 1;
+            for (int p = 0; p < rw.deg; ++p) nbar += c_new[prog.pos_in[rw.pos_base + p]];
+            float scale, fill;
+            worker_factors(a, n, nbar, scale, fill);
+            factors[j * n + w] = make_float2(scale, fill);
+        }
+    }
+    const int64_t nblk = (a.nquads + qb - 1) / qb;
+    for (int64_t b = blockIdx.x; b < nblk; b += gridDim.x) {
+        const int64_t q = b * qb + qi;
+        const bool active = q < a.nquads;
+        // m^{t0-1} of this CTA's quads (coalesced rows of qb quads) into buffer 1
+        for (int idx = tid; idx < E * qb; idx += blockDim.x) {
+            const int e = idx / qb;
+            const int64_t qg = b * qb + (idx - e * qb);
+            fused_mem[E * qb + idx] = qg < a.nquads ? ld_stream(a.msg_in + e * a.ld_m + 4 * qg) : zero;
+        }
+        float4 xv = zero, mv = zero, m1 = zero, m2 = zero;
+        if (active) {
+            xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
+            mv = (OBJ == relaysum::kMuStored) ? ld_stream(a.mu + i * a.ld_x + 4 * q)
+                                               : centre<kObj>(obj, mu_key, a, i, q, nullptr, 0);
+            if (OPT >= 1) m1 = *reinterpret_cast<const float4*>(a.s1 + i * a.ld_x + 4 * q);
+            if (OPT == 2) m2 = *reinterpret_cast<const float4*>(a.s2 + i * a.ld_x + 4 * q);
+        }
+        __syncthreads();
+        for (int j = 0; j < fs.k; ++j) {
+            float4* const cur = fused_mem + (j & 1) * E * qb + qi;
+            const float4* const prev = fused_mem + ((j + 1) & 1) * E * qb + qi;
+            float4 xh = zero;
+            if (active) {
+                const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i),
+                                         a.step + static_cast<uint32_t>(j), 0u, a.key);
+                const float st = fs.adam_step[j], ib = fs.adam_ibc2[j];
+                xh = relayed_with(a, xv, mv, z, [&](float4 g) { return update_rule<OPT>(a, st, ib, g, m1, m2); });
+                float* const out = (E > 0 && j + 2 >= fs.k) ? fs.msg[(j + 1) & 1] + 4 * q : nullptr;
+                switch (r.deg) {
+                    case 0: break;
+                    case 1: fused_small<1>(prog, r, a, xh, prev, cur, qb, out); break;
+                    case 2: fused_small<2>(prog, r, a, xh, prev, cur, qb, out); break;
+                    case 3: fused_small<3>(prog, r, a, xh, prev, cur, qb, out); break;
+                    case 4: fused_small<4>(prog, r, a, xh, prev, cur, qb, out); break;
+                    default: fused_wide(prog, r, a, xh, prev, cur, qb, out); break;
+                }
+            }
+            __syncthreads();
+            if (active) {
+                const float2 f = factors[j * n + i];  // (scale, fill)
+                float4 acc = xh;
+                if (f.y != 0.0f) acc = add4(scale4(xv, f.y), xh);
+                for (int k = 0; k < r.deg; ++k) acc = add4(acc, cur[prog.rb_in[r.pos_base + k] * qb]);
+                xv = scale4(acc, f.x);
+            }
+        }
+        if (active) {
+            st_stream(a.x + i * a.ld_x + 4 * q, xv);
+            if (OPT >= 1) st_stream(a.s1 + i * a.ld_x + 4 * q, m1);
+            if (OPT == 2) st_stream(a.s2 + i * a.ld_x + 4 * q, m2);
+        }
+        __syncthreads();  // the next block refills buffer 1
+    }
+}
+
 // --------------------------------------------------------------------- init
 
 __global__ void relay_init_kernel(float* x, float* msg_a, float* msg_b, int n, int E, int64_t ld_x,
@@ -821,16 +1032,31 @@ int models_threads(int nslots) {
     return t;
 }
 
-// Opts `Kernel` in to the full dynamic shared memory once per device and
-// returns its resident CTAs per SM for (threads, smem).  Both are cached per
-// device (queried once, not per step: steps may be captured into CUDA
-// graphs); each kernel instantiation has its own cache.  0 on a CUDA error.
+// Opts `Kernel` in to the dynamic shared memory it may use (kMaxSmem, less
+// when its static shared memory and kMaxSmem would pass the device's per-CTA
+// limit) once per device, and returns its resident CTAs per SM for
+// (threads, smem).  Both are cached per device (queried once, not per step:
+// steps may be captured into CUDA graphs); each kernel instantiation has its
+// own cache.  0 on a CUDA error, which is cleared so that it is not reported
+// again by a later launch.
 template <auto Kernel>
 int resident_ctas(int dev, int threads, size_t smem) {
     static std::atomic<bool> smem_set[kMaxDevices];
     if (dev >= kMaxDevices || !smem_set[dev].load()) {
-        if (cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) != cudaSuccess)
+        cudaFuncAttributes fa;
+        int optin = 0;
+        if (cudaFuncGetAttributes(&fa, Kernel) != cudaSuccess ||
+            cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) {
+            (void)cudaGetLastError();
             return 0;
+        }
+        const int room = optin - static_cast<int>(fa.sharedSizeBytes);
+        if (room <= 0 ||
+            cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 room < kMaxSmem ? room : kMaxSmem) != cudaSuccess) {
+            (void)cudaGetLastError();
+            return 0;
+        }
         if (dev < kMaxDevices) smem_set[dev].store(true);
     }
     static std::atomic<int64_t> occ_cache[kMaxDevices];
@@ -838,8 +1064,10 @@ int resident_ctas(int dev, int threads, size_t smem) {
     const int64_t cached = dev < kMaxDevices ? occ_cache[dev].load() : 0;
     if (cached != 0 && (cached >> 8) == key) return static_cast<int>(cached & 0xFF);
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, Kernel, threads, smem) != cudaSuccess || per_sm <= 0)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, Kernel, threads, smem) != cudaSuccess || per_sm <= 0) {
+        (void)cudaGetLastError();
         return 0;
+    }
     if (dev < kMaxDevices) occ_cache[dev].store((key << 8) | (per_sm & 0xFF));
     return per_sm;
 }
@@ -913,6 +1141,55 @@ int launch_models_obj(const relay_handle* h, const ModelArgs& a, cudaStream_t st
         case relaysum::kMuPerRow: return launch_models<relaysum::kMuPerRow, OPT>(h, a, stream, after_counts);
         default: return launch_models<relaysum::kMuCachedCentres, OPT>(h, a, stream, after_counts);
     }
+}
+
+// Quads per CTA of relay_fused_steps_kernel: nodes_qb, halved (down to 4)
+// while that leaves fewer CTAs than SMs, so short vectors still spread over
+// the whole GPU.
+int fused_qb(int n, int64_t nquads, int sms) {
+    int qb = nodes_qb(n);
+    while (qb > 4 && (nquads + qb - 1) / qb < sms) qb /= 2;
+    return qb;
+}
+
+template <int OBJ, int OPT>
+int launch_fused(const relay_handle* h, const ModelArgs& a, const FusedSteps& fs, cudaStream_t stream) {
+    int dev = 0;
+    const int sms = device_sms(&dev);
+    if (sms <= 0) return RELAY_ECUDA;
+    const int qb = fused_qb(h->prog.n, a.nquads, sms);
+    const int threads = qb * h->prog.n;
+    const size_t smem = static_cast<size_t>(2) * h->prog.E * qb * 16 + static_cast<size_t>(fs.k) * h->prog.n * 8;
+    if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
+    const int per_sm = resident_ctas<relay_fused_steps_kernel<OBJ, OPT>>(dev, threads, smem);
+    if (per_sm <= 0) return RELAY_ECUDA;
+    const int64_t want = (a.nquads + qb - 1) / qb;
+    const int64_t cap = static_cast<int64_t>(sms) * per_sm;
+    const int grid = static_cast<int>(want < cap ? want : cap);
+    const PhiloxKey mu_key = philox_key(static_cast<uint64_t>(h->obj.k0) | (static_cast<uint64_t>(h->obj.k1) << 32));
+    relay_fused_steps_kernel<OBJ, OPT><<<grid, threads, smem, stream>>>(h->prog, h->obj, mu_key, a, fs, qb);
+    return launch_status();
+}
+
+// relay_steps takes the fused kernel unless the walk is forced or, under
+// AUTO, a worker has more than kRegDeg neighbours: its threads then carry
+// all its edges at every step while the rest of the CTA waits at the
+// barrier (a 64-worker star measured 3.7x slower than one relay_step per
+// step).  Measured on one GB300 with every degree <= kRegDeg, from 8 workers
+// and d = 4096 to 32 workers and d = 1.1e8, the fused kernel was ahead
+// everywhere (1.2x to 1.8x).
+bool use_fused(const relay_handle* h) {
+    if (h->kernel == RELAY_KERNEL_NODES) return true;
+    if (h->kernel == RELAY_KERNEL_WALK) return false;
+    for (int i = 0; i < h->prog.n; ++i)
+        if (h->prog.node[i].deg > kRegDeg) return false;
+    return true;
+}
+
+template <int OPT>
+int launch_fused_obj(const relay_handle* h, const ModelArgs& a, const FusedSteps& fs, cudaStream_t stream) {
+    if (h->obj.source == relaysum::kMuStored) return launch_fused<relaysum::kMuStored, OPT>(h, a, fs, stream);
+    return launch_fused<relaysum::kMuPerRow, OPT>(h, a, fs, stream);
 }
 
 // Argument checks shared by relay_step_models and relay_step.
@@ -1160,14 +1437,19 @@ int relay_step_counts(relay_handle* h, int32_t* counts, relay_stream_t stream) {
     return launch_status();
 }
 
-// The step kernel's launch; `after_counts`: relay_step's counter kernel was
-// just enqueued on `stream`, so the step may start as its programmatic
-// dependent.
-static int step_models(relay_handle* h, float* x, const float* msg_in, float* msg_out, const int32_t* counts,
-                       float lr, uint64_t seed, int64_t step, relay_stream_t stream, bool after_counts) {
-    const int rc = check_step_args(h, x, msg_in, msg_out, counts, lr, step);
-    if (rc != RELAY_OK) return rc;
-    if (h->d == 0) return RELAY_OK;
+// Adam's bias-corrected factors of step t (k = t + 1), in double.
+static void adam_factors(const relay_handle* h, float lr, int64_t step, float* adam_step, float* adam_ibc2) {
+    *adam_step = 0.0f;
+    *adam_ibc2 = 0.0f;
+    if (h->opt != 2) return;
+    const double k = static_cast<double>(step) + 1.0;
+    *adam_step = static_cast<float>(lr / (1.0 - std::pow(static_cast<double>(h->beta1), k)));
+    *adam_ibc2 = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(static_cast<double>(h->beta2), k)));
+}
+
+// The step kernels' arguments for step `step` (checked by check_step_args).
+static ModelArgs model_args(const relay_handle* h, float* x, const float* msg_in, float* msg_out,
+                            const int32_t* counts, float lr, uint64_t seed, int64_t step) {
     ModelArgs a;
     a.x = x;
     a.mu = h->mu;
@@ -1191,13 +1473,19 @@ static int step_models(relay_handle* h, float* x, const float* msg_in, float* ms
     a.beta1 = h->beta1;
     a.beta2 = h->beta2;
     a.eps = h->eps;
-    a.adam_step = 0.0f;
-    a.adam_ibc2 = 0.0f;
-    if (h->opt == 2) {  // bias corrections of step k = t + 1, in double
-        const double k = static_cast<double>(step) + 1.0;
-        a.adam_step = static_cast<float>(lr / (1.0 - std::pow(static_cast<double>(h->beta1), k)));
-        a.adam_ibc2 = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(static_cast<double>(h->beta2), k)));
-    }
+    adam_factors(h, lr, step, &a.adam_step, &a.adam_ibc2);
+    return a;
+}
+
+// The step kernel's launch; `after_counts`: relay_step's counter kernel was
+// just enqueued on `stream`, so the step may start as its programmatic
+// dependent.
+static int step_models(relay_handle* h, float* x, const float* msg_in, float* msg_out, const int32_t* counts,
+                       float lr, uint64_t seed, int64_t step, relay_stream_t stream, bool after_counts) {
+    const int rc = check_step_args(h, x, msg_in, msg_out, counts, lr, step);
+    if (rc != RELAY_OK) return rc;
+    if (h->d == 0) return RELAY_OK;
+    const ModelArgs a = model_args(h, x, msg_in, msg_out, counts, lr, seed, step);
     switch (h->opt) {
         case 0: return launch_models_obj<0>(h, a, stream, after_counts);
         case 1: return launch_models_obj<1>(h, a, stream, after_counts);
@@ -1222,6 +1510,57 @@ int relay_step(relay_handle* h, float* x, const float* msg_in, float* msg_out, i
     rc = relay_step_counts(h, counts, stream);
     if (rc != RELAY_OK) return rc;
     return step_models(h, x, msg_in, msg_out, counts, lr, seed, step, stream, counted);
+}
+
+int relay_get_steps_kernel(const relay_handle* h) {
+    if (!h) return RELAY_EINVAL;
+    return use_fused(h) ? RELAY_KERNEL_FUSED : relay_get_kernel(h);
+}
+
+int relay_steps(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* counts, float lr, uint64_t seed,
+                int64_t t0, int64_t k, relay_stream_t stream) {
+    int rc = check_step_args(h, x, msg_a, msg_b, counts, lr, t0);
+    if (rc != RELAY_OK) return rc;
+    if (k < 0 || k > (int64_t(1) << 32) - t0) return RELAY_EINVAL;  // step counters stay below 2^32
+    float* const buf[2] = {msg_a, msg_b};
+    if (!use_fused(h)) {  // a wide node would hold its CTA at every step: one relay_step per step
+        for (int64_t j = 0; j < k; ++j) {
+            rc = relay_step(h, x, buf[j & 1], buf[(j + 1) & 1], counts, lr, seed, t0 + j, stream);
+            if (rc != RELAY_OK) return rc;
+        }
+        return RELAY_OK;
+    }
+    const bool counted = h->prog.E > 0 || h->algo == RELAY_ALGO_DME;
+    LostMask lost;
+    std::memcpy(lost.w, h->lost, sizeof(lost.w));
+    for (int64_t done = 0; done < k;) {
+        const int kc = static_cast<int>(k - done < kMaxFusedSteps ? k - done : kMaxFusedSteps);
+        const int par = static_cast<int>(done & 1);  // step t0 + done reads buf[par]
+        if (h->d > 0) {
+            const ModelArgs a = model_args(h, x, buf[par], buf[par ^ 1], counts, lr, seed, t0 + done);
+            FusedSteps fs;
+            fs.k = kc;
+            fs.msg[0] = buf[par];
+            fs.msg[1] = buf[par ^ 1];
+            for (int j = 0; j < kMaxFusedSteps; ++j)
+                adam_factors(h, lr, t0 + done + (j < kc ? j : 0), &fs.adam_step[j], &fs.adam_ibc2[j]);
+            switch (h->opt) {
+                case 0: rc = launch_fused_obj<0>(h, a, fs, stream); break;
+                case 1: rc = launch_fused_obj<1>(h, a, fs, stream); break;
+                default: rc = launch_fused_obj<2>(h, a, fs, stream); break;
+            }
+            if (rc != RELAY_OK) return rc;
+        }
+        // the counters advance after the models kernel, which read them
+        if (counted) {
+            relay_counts_steps_kernel<<<1, 256, 0, stream>>>(h->prog, lost, h->has_lost ? 1 : 0, counts,
+                                                             h->algo == RELAY_ALGO_DME ? h->dme_count : nullptr, kc);
+            rc = launch_status();
+            if (rc != RELAY_OK) return rc;
+        }
+        done += kc;
+    }
+    return RELAY_OK;
 }
 
 int relay_nbar(const relay_handle* h, const int32_t* counts_host, int32_t* nbar_host) {

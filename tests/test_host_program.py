@@ -297,6 +297,15 @@ def test_create_limits_and_layout():
         with pytest.raises(rs.RelayError) as e:
             rs.relay_set_kernel(h, k)
         assert e.value.status == rs.RELAY_EINVAL
+    # relay_steps: the fused kernel unless the walk is forced or (AUTO) a node is wide
+    for tree, auto in ((wl.chain(8), rs.RELAY_KERNEL_FUSED), (wl.binary_tree(8), rs.RELAY_KERNEL_FUSED),
+                       (wl.star(8), rs.RELAY_KERNEL_WALK)):
+        hs = rs.relay_create(8, 1 << 24, tree)
+        assert rs.relay_get_steps_kernel(hs) == auto
+        rs.relay_set_kernel(hs, rs.RELAY_KERNEL_NODES)
+        assert rs.relay_get_steps_kernel(hs) == rs.RELAY_KERNEL_FUSED
+        rs.relay_set_kernel(hs, rs.RELAY_KERNEL_WALK)
+        assert rs.relay_get_steps_kernel(hs) == rs.RELAY_KERNEL_WALK
     with pytest.raises(rs.RelayError):
         rs.relay_set_coord_offset(h, 6)
     rs.relay_set_coord_offset(h, 8)
@@ -332,6 +341,15 @@ def test_step_rejects_bad_arguments_before_any_launch():
     assert lib.relay_step(h.raw, fake, big, 2 * big, fake, float("nan"), 0, 0, None) == rs.RELAY_EINVAL
     assert lib.relay_step(h.raw, fake, fake + 256, 2 * big, fake, 0.1, 0, 0, None) == rs.RELAY_EINVAL
     assert lib.relay_step(h.raw, fake, big, 2 * big, fake, 0.1, 0, 1 << 32, None) == rs.RELAY_EINVAL
+    # relay_steps: the same checks, plus k >= 0 and t0 + k <= 2^32
+    lib.relay_steps.argtypes = [ctypes.c_void_p] * 5 + [ctypes.c_float, ctypes.c_uint64, ctypes.c_int64,
+                                                        ctypes.c_int64, ctypes.c_void_p]
+    assert lib.relay_steps(h.raw, fake, big, big, fake, 0.1, 0, 0, 1, None) == rs.RELAY_EINVAL
+    assert lib.relay_steps(h.raw, fake, big, 2 * big, fake, 0.1, 0, -1, 1, None) == rs.RELAY_EINVAL
+    assert lib.relay_steps(h.raw, fake, big, 2 * big, fake, float("inf"), 0, 0, 1, None) == rs.RELAY_EINVAL
+    assert lib.relay_steps(h.raw, fake, big, 2 * big, fake, 0.1, 0, 0, -1, None) == rs.RELAY_EINVAL
+    assert lib.relay_steps(h.raw, fake, big, 2 * big, fake, 0.1, 0, 5, (1 << 32) - 4, None) == rs.RELAY_EINVAL
+    assert lib.relay_steps(h.raw, fake, big, 2 * big, fake, 0.1, 0, 0, 0, None) == rs.RELAY_OK  # nothing to do
 
 
 def test_binding_fails_loudly_without_the_library(monkeypatch, tmp_path):
