@@ -3,8 +3,9 @@
  * compares the models it writes with the Python binding's run of the same
  * configuration.
  *
- * usage: c_abi_run <tree: chain|binary> <n> <d> <steps> <mode> <out.bin>
- * writes x (float32 [n][d]) and the two metrics (double [2]) to out.bin. */
+ * usage: c_abi_run <tree: chain|binary> <n> <d> <steps> <mode> <out.bin> [fused]
+ * writes x (float32 [n][d]) and the two metrics (double [2]) to out.bin; with
+ * "fused" the steps run as one relay_steps call instead of relay_step calls. */
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -32,10 +33,11 @@
     } while (0)
 
 int main(int argc, char **argv) {
-    if (argc != 7) {
-        fprintf(stderr, "usage: %s chain|binary n d steps mode out.bin\n", argv[0]);
+    if (argc != 7 && !(argc == 8 && strcmp(argv[7], "fused") == 0)) {
+        fprintf(stderr, "usage: %s chain|binary n d steps mode out.bin [fused]\n", argv[0]);
         return 2;
     }
+    const int fused = argc == 8;
     const int binary = strcmp(argv[1], "binary") == 0;
     const int n = atoi(argv[2]);
     const int64_t d = atoll(argv[3]);
@@ -80,8 +82,12 @@ int main(int argc, char **argv) {
     CHECK(relay_fill_objective(h, mu, mix, n, 2.0f, mu_seed, s));
     CHECK(relay_set_objective(h, mu, sigma));
     CHECK(relay_init(h, x, msg[0], msg[1], counts, 0.0f, seed, s));
-    for (int64_t t = 0; t < steps; ++t)
-        CHECK(relay_step(h, x, msg[t & 1], msg[(t + 1) & 1], counts, lr, seed, t, s));
+    if (fused) {
+        CHECK(relay_steps(h, x, msg[0], msg[1], counts, lr, seed, 0, steps, s));
+    } else {
+        for (int64_t t = 0; t < steps; ++t)
+            CHECK(relay_step(h, x, msg[t & 1], msg[(t + 1) & 1], counts, lr, seed, t, s));
+    }
     CHECK(relay_metrics_static(h, x, out, s));
     CUDA(cudaStreamSynchronize(stream));
 
