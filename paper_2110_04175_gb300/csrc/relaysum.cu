@@ -713,7 +713,8 @@ struct FusedSteps {
 // They go to `cur`, and to HBM at `out` (row e at out + e * ld_m) unless null.
 template <int D>
 __device__ __forceinline__ void fused_small(const Program& prog, const NodeRec& r, const ModelArgs& a, float4 xh,
-                                            const float4* prev, float4* cur, int qb, float* out) {
+                                            const float4* prev, float4* cur, int qb, float* out,
+                                            uint32_t lost_bits) {
     float4 m[D];
 #pragma unroll
     for (int s = 0; s < D; ++s) m[s] = prev[prog.pos_in[r.pos_base + s] * qb];
@@ -728,10 +729,20 @@ __device__ __forceinline__ void fused_small(const Program& prog, const NodeRec& 
 #pragma unroll
     for (int s = 0; s < D; ++s) {
         const int e = prog.pos_out[r.pos_base + s];
-        const float4 o = delivered(a, e, (s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]));
+        const float4 o = ((lost_bits >> s) & 1u) ? make_float4(0.f, 0.f, 0.f, 0.f)
+                                                 : ((s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]));
         cur[e * qb] = o;
         if (out) st_stream(out + e * a.ld_m, o);
     }
+}
+
+// The rebuild sum: acc plus the incoming messages of step j in rb_in order.
+template <int D>
+__device__ __forceinline__ float4 fused_rebuild(const Program& prog, const NodeRec& r, const float4* cur, int qb,
+                                                float4 acc) {
+#pragma unroll
+    for (int k = 0; k < D; ++k) acc = add4(acc, cur[prog.rb_in[r.pos_base + k] * qb]);
+    return acc;
 }
 
 __device__ __noinline__ void fused_wide(const Program& prog, const NodeRec& r, const ModelArgs& a, float4 xh,
@@ -772,6 +783,10 @@ relay_fused_steps_kernel(const __grid_constant__ Program prog, const __grid_cons
     const NodeRec r = prog.node[i];
     const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
     float2* const factors = reinterpret_cast<float2*>(fused_mem + 2 * E * qb);  // [j * n + i]
+    // bit s: the message to this worker's neighbour s is lost (narrow nodes)
+    uint32_t lost_bits = 0;
+    if (a.has_lost && r.deg <= kRegDeg)
+        for (int s = 0; s < r.deg; ++s) lost_bits |= (a.lost(prog.pos_out[r.pos_base + s]) ? 1u : 0u) << s;
     for (int e = tid; e < E; e += blockDim.x) c_mem[1][e] = a.counts[e];  // c^{t0-1}
     __syncthreads();
     for (int j = 0; j < fs.k; ++j) {
@@ -819,10 +834,10 @@ relay_fused_steps_kernel(const __grid_constant__ Program prog, const __grid_cons
                 float* const out = (E > 0 && j + 2 >= fs.k) ? fs.msg[(j + 1) & 1] + 4 * q : nullptr;
                 switch (r.deg) {
                     case 0: break;
-                    case 1: fused_small<1>(prog, r, a, xh, prev, cur, qb, out); break;
-                    case 2: fused_small<2>(prog, r, a, xh, prev, cur, qb, out); break;
-                    case 3: fused_small<3>(prog, r, a, xh, prev, cur, qb, out); break;
-                    case 4: fused_small<4>(prog, r, a, xh, prev, cur, qb, out); break;
+                    case 1: fused_small<1>(prog, r, a, xh, prev, cur, qb, out, lost_bits); break;
+                    case 2: fused_small<2>(prog, r, a, xh, prev, cur, qb, out, lost_bits); break;
+                    case 3: fused_small<3>(prog, r, a, xh, prev, cur, qb, out, lost_bits); break;
+                    case 4: fused_small<4>(prog, r, a, xh, prev, cur, qb, out, lost_bits); break;
                     default: fused_wide(prog, r, a, xh, prev, cur, qb, out); break;
                 }
             }
@@ -831,7 +846,16 @@ relay_fused_steps_kernel(const __grid_constant__ Program prog, const __grid_cons
                 const float2 f = factors[j * n + i];  // (scale, fill)
                 float4 acc = xh;
                 if (f.y != 0.0f) acc = add4(scale4(xv, f.y), xh);
-                for (int k = 0; k < r.deg; ++k) acc = add4(acc, cur[prog.rb_in[r.pos_base + k] * qb]);
+                switch (r.deg) {
+                    case 0: break;
+                    case 1: acc = fused_rebuild<1>(prog, r, cur, qb, acc); break;
+                    case 2: acc = fused_rebuild<2>(prog, r, cur, qb, acc); break;
+                    case 3: acc = fused_rebuild<3>(prog, r, cur, qb, acc); break;
+                    case 4: acc = fused_rebuild<4>(prog, r, cur, qb, acc); break;
+                    default:
+                        for (int k = 0; k < r.deg; ++k) acc = add4(acc, cur[prog.rb_in[r.pos_base + k] * qb]);
+                        break;
+                }
                 xv = scale4(acc, f.x);
             }
         }
