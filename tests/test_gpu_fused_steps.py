@@ -163,3 +163,32 @@ def test_steps_against_oracle(shape, n, d, mode):
     assert parity_error(run.x[:, :d].double().cpu().numpy(), st.x) <= RTOL
     assert parity_error(run.messages[:run.E, :d].double().cpu().numpy(), st.msg) <= RTOL
     assert np.array_equal(run.counts[:run.E].cpu().numpy(), st.counts)
+
+
+@pytest.mark.parametrize("name", ["chain16_d9231114_dirichlet", "binary32_d110000000"])
+def test_full_size_steps_equal_step_calls(name):
+    """At the sizes bench.py times, every CTA of the fused kernel carries
+    hundreds of quad blocks in turn (its loop refills the message buffer and
+    reuses the rebuild factors), which the small cases above never reach:
+    70 steps (two launches) through relay_steps equal 70 relay_step calls bit
+    for bit there too -- models, both message buffers and counters."""
+    w = wl.by_name(name)
+    runs = []
+    for _ in range(2):
+        run = rs.RelayRun(w.n, w.d, w.edges, device="cuda:0", mode=w.mode)
+        run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+        runs.append(run)
+    a, b = runs
+    assert rs.relay_get_steps_kernel(b.h) == rs.RELAY_KERNEL_FUSED
+    for _ in range(70):
+        a.step(w.lr, w.seed)
+    b.steps(70, w.lr, w.seed)
+    torch.cuda.synchronize()
+    assert torch.equal(a.x[:, :w.d], b.x[:, :w.d])
+    for k in (0, 1):
+        assert torch.equal(a.msg[k][:a.E, :w.d], b.msg[k][:b.E, :w.d]), k
+    assert torch.equal(a.counts[:a.E], b.counts[:b.E])
+    assert a.cur == b.cur
+    del a, b, runs
+    gc.collect()
+    torch.cuda.empty_cache()
