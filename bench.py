@@ -653,6 +653,21 @@ def run_e2e(args, w, run, dev, stream, world: int):
     host.sync()
     ms = reduce_max((time.perf_counter() - t0) * 1e3, world)
     h2d, d2h = host.bytes_per_step()
+    fused = None
+    if args.fused_steps > 0:
+        # the same host-state path with relay_steps: the state crosses the
+        # link once per call of K steps (one relay_steps call per chunk visit)
+        K = args.fused_steps
+        host.steps(2, w.lr, w.seed)
+        host.sync()
+        barrier(world)
+        t1 = time.perf_counter()
+        host.steps(K, w.lr, w.seed)
+        host.sync()
+        fms = reduce_max((time.perf_counter() - t1) * 1e3, world)
+        fused = {"value": round(world * K / (fms / 1e3), 4), "unit": "steps/s", "steps_per_call": K,
+                 "h2d_bytes_per_call": h2d, "d2h_bytes_per_call": d2h,
+                 "note": "HostRelayRun.steps: one relay_steps call per chunk visit"}
     return {"value": round(world * args.e2e_steps / (ms / 1e3), 4), "unit": "steps/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
             "path": "HostRelayRun: state in pinned host memory, streamed through the GPU in "
@@ -661,7 +676,8 @@ def run_e2e(args, w, run, dev, stream, world: int):
                     "x, the counters and the message rows a later step reads cross the link",
             "copy_gbs": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9, 1),
             "host_link": link,
-            "copy_frac": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9 / link["both_gbs"], 3)}
+            "copy_frac": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9 / link["both_gbs"], 3),
+            "fused_steps": fused}
 
 
 def traffic_per_launch(w, objective: str, kernel: str = "relay_models_kernel", optimizer: str = "sgd"):

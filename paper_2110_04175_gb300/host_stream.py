@@ -13,6 +13,10 @@ one contiguous block).  A step:
    device-to-host copies -- so both copy directions and the kernels overlap;
 3. copies the counters out.
 
+``steps(k)`` instead runs k steps per chunk visit (one relay_steps call per
+chunk, the counters restored before each), so the state crosses the link
+once per k steps.
+
 Only the message rows that a later step reads cross the link.  A message
 arriving at a leaf is consumed by the leaf's rebuild in the step that forms
 it (a leaf's only outgoing message excludes its only incoming one), so those
@@ -164,6 +168,55 @@ class HostRelayRun:
             self.counts_saved.record(self.s_out)
         self.cur = 1 - self.cur
         self.t += 1
+
+    def steps(self, k: int, lr: float, seed: int):
+        """Enqueues k steps with one relay_steps call per chunk visit, so the
+        state crosses the host link once per k steps instead of once per
+        step.  The counters are per edge, not per coordinate: every chunk's
+        call starts from the same c^{t-1}, restored from the host copy before
+        it, and the last chunk's result goes back.  Afterwards the host holds
+        x, the counters and m^{t+k-1} (the rows a later step reads), equal bit
+        for bit to k step() calls; the other message buffer is not kept."""
+        import torch
+        k = int(k)
+        if k <= 0:
+            return
+        src, dst = self.msg_h[self.cur], self.msg_h[self.cur ^ (k & 1)]
+        with torch.cuda.stream(self.s_comp):
+            self.s_comp.wait_event(self.counts_saved)
+        for c in range(self.nchunks):
+            b = c % self.B
+            s_in = self.s_ins[c % len(self.s_ins)]
+            s_out = self.s_outs[c % len(self.s_outs)]
+            final = self.mob[b] if k & 1 else self.mib[b]  # the buffer step t+k-1 writes
+            with torch.cuda.stream(s_in):
+                s_in.wait_event(self.out_done[b])
+                s_in.wait_event(self.out_done_k[c])
+                self.xb[b].copy_(self.x_h[c], non_blocking=True)
+                for lo, hi in self.kept_runs:
+                    self.mib[b][lo:hi].copy_(src[c][lo:hi], non_blocking=True)
+                self.in_done[b].record(s_in)
+            with torch.cuda.stream(self.s_comp):
+                self.s_comp.wait_event(self.in_done[b])
+                self.counts_d.copy_(self.counts_h, non_blocking=True)
+                nat.relay_steps(self._handle(c), self.xb[b], self.mib[b], self.mob[b], self.counts_d, lr, seed,
+                                self.t, k, self.s_comp)
+                self.comp_done[b].record(self.s_comp)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(self.comp_done[b])
+                self.x_h[c].copy_(self.xb[b], non_blocking=True)
+                for lo, hi in self.kept_runs:
+                    dst[c][lo:hi].copy_(final[lo:hi], non_blocking=True)
+                self.out_done[b].record(s_out)
+                self.out_done_k[c].record(s_out)
+        with torch.cuda.stream(self.s_comp):
+            self.counts_ready.record(self.s_comp)
+        with torch.cuda.stream(self.s_out):
+            self.s_out.wait_event(self.counts_ready)
+            self.counts_h.copy_(self.counts_d, non_blocking=True)
+            self.counts_saved.record(self.s_out)
+        self.cur ^= k & 1
+        self.t += k
 
     def sync(self):
         import torch
