@@ -226,7 +226,7 @@ int relay_step(relay_handle *h, float *x, const float *msg_in, float *msg_out,
  * evolves on its own, so the steps run without a round trip through HBM:
  * each CTA keeps its quads' models and optimiser state in registers and
  * their messages in shared memory for up to 64 steps per launch (then a
- * 1-CTA launch advances the counters).  That fused kernel is taken under
+ * 1-CTA launch advances the counters).  That multi-step kernel is taken under
  * RELAY_KERNEL_NODES, and under RELAY_KERNEL_AUTO when no worker has more
  * than 4 neighbours; otherwise (RELAY_KERNEL_WALK, or a wide node such as a
  * star's hub, whose threads would hold their CTA at every step) relay_steps

@@ -1195,12 +1195,12 @@ int launch_fused(const relay_handle* h, const ModelArgs& a, const FusedSteps& fs
     return launch_status();
 }
 
-// relay_steps takes the fused kernel unless the walk is forced or, under
+// relay_steps takes the multi-step kernel unless the walk is forced or, under
 // AUTO, a worker has more than kRegDeg neighbours: its threads then carry
 // all its edges at every step while the rest of the CTA waits at the
 // barrier (a 64-worker star measured 3.7x slower than one relay_step per
 // step).  Measured on one GB300 with every degree <= kRegDeg, from 8 workers
-// and d = 4096 to 32 workers and d = 1.1e8, the fused kernel was ahead
+// and d = 4096 to 32 workers and d = 1.1e8, the multi-step kernel was ahead
 // everywhere (1.2x to 1.8x).
 bool use_fused(const relay_handle* h) {
     if (h->kernel == RELAY_KERNEL_NODES) return true;

@@ -90,7 +90,7 @@ def state_of(run):
 @pytest.mark.parametrize("kernel", ["auto", "nodes"])
 @pytest.mark.parametrize("name", sorted(CASES))
 def test_steps_equal_step_calls_bit_for_bit(name, kernel):
-    """kernel="nodes" forces the fused kernel for relay_steps (the wide-node
+    """kernel="nodes" forces the multi-step kernel for relay_steps (the wide-node
     path included) and the node kernel for relay_step; under "auto" the stars
     take the per-step fallback and the walk."""
     c = CASES[name]
@@ -167,7 +167,7 @@ def test_steps_against_oracle(shape, n, d, mode):
 
 @pytest.mark.parametrize("name", ["chain16_d9231114_dirichlet", "binary32_d110000000"])
 def test_full_size_steps_equal_step_calls(name):
-    """At the sizes bench.py times, every CTA of the fused kernel carries
+    """At the sizes bench.py times, every CTA of the multi-step kernel carries
     hundreds of quad blocks in turn (its loop refills the message buffer and
     reuses the rebuild factors), which the small cases above never reach:
     70 steps (two launches) through relay_steps equal 70 relay_step calls bit

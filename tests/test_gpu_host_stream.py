@@ -51,7 +51,7 @@ def test_host_stream_equals_resident_run(shape, n, d, chunk, buffers):
 
 
 @pytest.mark.parametrize("shape,n,d,chunk,buffers", [
-    ("binary", 16, 1_000_003, 1 << 18, 3),   # 4 chunks, fused kernel
+    ("binary", 16, 1_000_003, 1 << 18, 3),   # 4 chunks, multi-step kernel
     ("star", 12, 70_001, 1 << 14, 2),        # wide node: relay_steps repeats relay_step
     ("chain", 5, 1_000, 1 << 12, 3),         # a single chunk
     ("pair", 2, 5_000, 1 << 12, 2),          # no message row kept

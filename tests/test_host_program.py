@@ -297,7 +297,7 @@ def test_create_limits_and_layout():
         with pytest.raises(rs.RelayError) as e:
             rs.relay_set_kernel(h, k)
         assert e.value.status == rs.RELAY_EINVAL
-    # relay_steps: the fused kernel unless the walk is forced or (AUTO) a node is wide
+    # relay_steps: the multi-step kernel unless the walk is forced or (AUTO) a node is wide
     for tree, auto in ((wl.chain(8), rs.RELAY_KERNEL_FUSED), (wl.binary_tree(8), rs.RELAY_KERNEL_FUSED),
                        (wl.star(8), rs.RELAY_KERNEL_WALK)):
         hs = rs.relay_create(8, 1 << 24, tree)
