@@ -25,6 +25,7 @@ the CPU oracle instead (rank 0 only).
 from __future__ import annotations
 
 import argparse
+import gc
 import json
 import os
 import statistics
@@ -336,36 +337,35 @@ def workload_config(w, gpus: int, args=None, dev=None) -> dict:
 
 # ------------------------------------------------------------------ native
 
-def run_native(args, w, rank: int, world: int):
+def make_run(args, w, dev, c0: int):
+    """The resident run of workload `w` on `dev`, initialised (RelayRun owns
+    the buffers; the library's kernels do all the work)."""
+    import paper_2110_04175_gb300 as rs
+    optimizer = {"sgd": None, "nesterov": ("nesterov", 0.9),
+                 "adam": ("adam", 0.9, 0.999, 1e-8)}[args.optimizer]
+    run = rs.RelayRun(w.n, w.d, w.edges, device=dev, mode=w.mode, c0=c0, objective=args.objective,
+                      optimizer=optimizer, algorithm=args.algorithm, kernel=args.kernel)
+    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
+    return run
+
+
+def make_stepper(args, w, run, stream, rank: int):
+    """one_step(ev): one step of `run` on `stream`; ev (per tree window: three
+    CUDA events) brackets the counter kernel and the step kernel.  Several
+    tree windows (double binary trees) are one step, timed as a whole."""
     import numpy as np
     import torch
 
     import paper_2110_04175_gb300 as rs
 
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    stream = torch.cuda.current_stream(dev)
-    c0 = shard_offset(rank, w.d)
-    optimizer = {"sgd": None, "nesterov": ("nesterov", 0.9),
-                 "adam": ("adam", 0.9, 0.999, 1e-8)}[args.optimizer]
-    run = rs.RelayRun(w.n, w.d, w.edges, device=dev, mode=w.mode, c0=c0, objective=args.objective,
-                      optimizer=optimizer, algorithm=args.algorithm, kernel=args.kernel)
     lost_rng = np.random.default_rng(1234 + rank)
-    run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
-    h = run.h
-    kernel_name = ("relay_nodes_kernel" if rs.relay_get_kernel(h) == rs.RELAY_KERNEL_NODES
-                   else "relay_models_kernel")
 
     def one_step(ev=None):
         torch.cuda.nvtx.range_push(f"relay_step {run.t}")  # a named range per step for profilers
+        for tr in run.trees:
+            if args.lost_prob > 0:  # messages lost in transit this step (Section 4.4)
+                rs.relay_set_lost_messages(tr.h, lost_rng.random(tr.E) < args.lost_prob)
         if len(run.trees) > 1:
-            # several tree windows (double binary trees): RelayRun.step forks
-            # them onto their own streams and joins them back; the step is
-            # timed as a whole
-            for tr in run.trees:
-                if args.lost_prob > 0:
-                    rs.relay_set_lost_messages(tr.h, lost_rng.random(tr.E) < args.lost_prob)
             if ev is not None:
                 ev[0][0].record(stream)
                 ev[0][1].record(stream)
@@ -374,27 +374,28 @@ def run_native(args, w, rank: int, world: int):
                 ev[-1][2].record(stream)
             torch.cuda.nvtx.range_pop()
             return
-        for k, tr in enumerate(run.trees):
-            if args.lost_prob > 0:  # messages lost in transit this step (Section 4.4)
-                rs.relay_set_lost_messages(tr.h, lost_rng.random(tr.E) < args.lost_prob)
-            if ev is not None:
-                ev[k][0].record(stream)
-            rs.relay_step_counts(tr.h, tr.counts, stream)
-            if ev is not None:
-                ev[k][1].record(stream)
-            rs.relay_step_models(tr.h, run._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts,
-                                 w.lr, w.seed, run.t, stream)
-            if ev is not None:
-                ev[k][2].record(stream)
-            tr.cur = 1 - tr.cur
+        tr = run.trees[0]
+        if ev is not None:
+            ev[0][0].record(stream)
+        rs.relay_step_counts(tr.h, tr.counts, stream)
+        if ev is not None:
+            ev[0][1].record(stream)
+        rs.relay_step_models(tr.h, run._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts,
+                             w.lr, w.seed, run.t, stream)
+        if ev is not None:
+            ev[0][2].record(stream)
+        tr.cur = 1 - tr.cur
         run.t += 1
         torch.cuda.nvtx.range_pop()
 
+    return one_step
+
+
+def time_steps(args, w, run, one_step, dev, stream, rank: int, world: int, local: int):
+    """Times args.steps steps (after the warm-up already run): (total ms,
+    max over ranks; step-kernel ms of every step; clock summary)."""
+    import torch
     T = len(run.trees)
-    for _ in range(args.warmup):
-        one_step()
-    if args.graph:
-        return run_graphed(args, w, run, dev, stream, rank, world)
     # a working set that fits in L2 is evicted before every timed step (a
     # memset of twice the L2), and the steps are then timed one by one
     flush = None
@@ -418,23 +419,25 @@ def run_native(args, w, rank: int, world: int):
     else:
         total_ms = sum(events[k][0][0].elapsed_time(events[k][-1][2]) for k in range(args.steps))
         del flush
-    # step-kernel time per step (several windows: the whole forked step)
+    # step-kernel time per step (several windows: the whole step)
     if T == 1:
         models_ms = [events[k][0][1].elapsed_time(events[k][0][2]) for k in range(args.steps)]
     else:
         models_ms = [events[k][0][1].elapsed_time(events[k][-1][2]) for k in range(args.steps)]
-    total_ms = reduce_max(total_ms, world)
-    steps_per_s = world * args.steps / (total_ms / 1e3)
+    return reduce_max(total_ms, world), models_ms, clocks.summary()
 
-    # several steps per call, on the resident run (before run_e2e frees it)
-    fused = run_fused(args, w, run, dev, stream, world) if args.fused_steps > 0 else None
-    # end to end: state in pinned host memory, copied in and out every step
-    e2e = None
-    if args.e2e_steps > 0:
-        e2e = run_e2e(args, w, run, dev, stream, world)
 
-    if rank != 0:
-        return
+def kernel_name_of(run) -> str:
+    import paper_2110_04175_gb300 as rs
+    name = ("relay_nodes_kernel" if rs.relay_get_kernel(run.h) == rs.RELAY_KERNEL_NODES
+            else "relay_models_kernel")
+    T = len(run.trees)
+    return name if T == 1 else f"{name} on {T} tree windows, overlapped (whole step timed)"
+
+
+def roofline_of(args, w, run, models_ms) -> dict:
+    """The step kernel's algorithmic HBM bytes per launch over its mean
+    CUDA-event time, against the measured copy bandwidth."""
     peaks = measured_peaks()
     peak = peaks.get("hbm_gbs")
     peak_src = "measured" if peak else "fallback"
@@ -444,12 +447,12 @@ def run_native(args, w, rank: int, world: int):
     alg_bytes = w.bytes_per_step() + 4 * w.d * w.n * state_rows
     moved = alg_bytes if args.objective == "generated" else alg_bytes + 4 * w.d * w.n
     achieved = alg_bytes / (mean_models_ms / 1e3) / 1e9
+    name = kernel_name_of(run)
+    base = name.split(" ")[0]
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4),
-                "traffic": traffic_per_launch(w, args.objective, kernel_name, args.optimizer),
-                "kernel": kernel_name if T == 1 else
-                f"{kernel_name} on {T} tree windows, overlapped (whole step timed)",
-                "peak_source": peak_src,
+                "traffic": traffic_per_launch(w, args.objective, base, args.optimizer),
+                "kernel": name, "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "algorithmic_bytes_rule": "4 d (2n + 2E) [+ 4 d n x optimiser-state rows]",
                 "objective": args.objective,
@@ -463,6 +466,45 @@ def run_native(args, w, rank: int, world: int):
         # the ncu DRAM bytes of one launch over this run's mean launch time
         roofline["dram_gbs"] = round(roofline["traffic"] / (mean_models_ms / 1e3) / 1e9, 1)
         roofline["dram_frac"] = round(roofline["dram_gbs"] / peak, 4)
+    return roofline
+
+
+def run_native(args, w, rank: int, world: int):
+    import torch
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    c0 = shard_offset(rank, w.d)
+    run = make_run(args, w, dev, c0)
+    one_step = make_stepper(args, w, run, stream, rank)
+    T = len(run.trees)
+    for _ in range(args.warmup):
+        one_step()
+    if args.graph:
+        return run_graphed(args, w, run, dev, stream, rank, world)
+    total_ms, models_ms, clocks = time_steps(args, w, run, one_step, dev, stream, rank, world, local)
+    steps_per_s = world * args.steps / (total_ms / 1e3)
+    roofline = roofline_of(args, w, run, models_ms) if rank == 0 else None
+    alg_bytes = w.bytes_per_step()
+
+    # several steps per call, on the resident run (before run_e2e frees it)
+    fused = run_fused(args, w, run, dev, stream, world) if args.fused_steps > 0 else None
+    # end to end: state in pinned host memory, copied in and out every step
+    e2e = None
+    if args.e2e_steps > 0:
+        e2e = run_e2e(args, w, run, dev, stream, world)
+    del run, one_step
+    gc.collect()
+    torch.cuda.empty_cache()
+    # the other HBM-bound workloads, each timed like the headline
+    per_workload = None
+    if args.per_workload and args.d is None:
+        per_workload = run_per_workload(args, w, dev, stream, rank, world, local)
+
+    if rank != 0:
+        return
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         cpu = oracle_sample(w)
@@ -471,10 +513,48 @@ def run_native(args, w, rank: int, world: int):
             "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": workload_config(w, world, args, dev), "roofline": roofline, "cpu_baseline": cpu,
-            "e2e": e2e, "gpu_launches": 2 * T * args.steps, "clocks": clocks.summary(),
+            "e2e": e2e, "gpu_launches": 2 * T * args.steps, "clocks": clocks,
             "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1),
-            "fused_steps": fused}
+            "fused_steps": fused, "per_workload": per_workload}
     print(json.dumps(line), flush=True)
+
+
+PER_WORKLOAD = ["chain16_d9231114_dirichlet", "star64_d25000000", "chain64_d25000000",
+                "binary64_d25000000", "torus64_d25000000", "double16_d9231114"]
+
+
+def run_per_workload(args, head, dev, stream, rank: int, world: int, local: int) -> list:
+    """Each of the other HBM-bound workloads (the 16-worker VGG-11-sized chain
+    with Dirichlet centres; the four 64-worker trees at d = 2.5e7; the double
+    binary trees), timed as the headline is: a fresh resident run, the same
+    warm-up and step count, CUDA events on the launching stream, the clocks
+    sampled meanwhile.  Each run's buffers are freed before the next."""
+    import torch
+
+    from paper_2110_04175_gb300 import workloads as wl
+
+    out = []
+    for name in PER_WORKLOAD:
+        if name == head.name:
+            continue
+        w = wl.by_name(name)
+        run = make_run(args, w, dev, shard_offset(rank, w.d))
+        one_step = make_stepper(args, w, run, stream, rank)
+        for _ in range(args.warmup):
+            one_step()
+        total_ms, models_ms, clocks = time_steps(args, w, run, one_step, dev, stream, rank, world, local)
+        if rank == 0:
+            cfg = workload_config(w, world, args, dev)
+            out.append({"workload": name, "value": round(world * args.steps / (total_ms / 1e3), 4),
+                        "unit": "steps/s", "ms_per_step": round(total_ms / args.steps, 4),
+                        "n_workers": w.n, "tree": cfg["tree"], "d": w.d, "steps": args.steps,
+                        "warmup": args.warmup, "l2": cfg["l2"],
+                        "roofline": roofline_of(args, w, run, models_ms), "clocks": clocks,
+                        "gpu_launches": 2 * len(run.trees) * args.steps})
+        del run, one_step
+        gc.collect()
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_fused(args, w, run, dev, stream, world: int) -> dict:
@@ -511,9 +591,14 @@ def run_fused(args, w, run, dev, stream, world: int) -> dict:
     fused = all(rs.relay_get_steps_kernel(tr.h) == rs.RELAY_KERNEL_FUSED for tr in run.trees)
     E, state_rows = w.E, {"sgd": 0, "nesterov": 1, "adam": 2}[args.optimizer]
     mu_rows = w.n if args.objective == "stored" else 0
-    # per call: read x, mu, the state, m^{t0-1}; write x, the state and the last two steps' messages
-    per_call = 4 * w.d * (w.n + mu_rows + state_rows * w.n + E + w.n + state_rows * w.n + min(K, 2) * E)
-    launches = (-(-K // 64)) * (1 + (E > 0 or args.algorithm == "dme")) if fused else 2 * K
+    # per launch of at most 64 steps: read x, mu, the state, m^{t0-1}; write x, the state and
+    # the last two steps' messages
+    chunks = -(-K // 64)
+    per_call = 0
+    for j in range(chunks):
+        kc = min(64, K - 64 * j)
+        per_call += 4 * w.d * (w.n + mu_rows + state_rows * w.n + E + w.n + state_rows * w.n + min(kc, 2) * E)
+    launches = chunks * (1 + (E > 0 or args.algorithm == "dme")) if fused else 2 * K
     return {"value": round(world * K * calls / (ms / 1e3), 4), "unit": "steps/s", "steps_per_call": K,
             "calls": calls, "ms_per_step": round(ms / (K * calls), 5),
             "kernel": "relay_fused_steps_kernel" if fused else "one relay_step per step (a wide node)",
@@ -611,8 +696,11 @@ def host_link_gbs(dev, mib: int = 1024, reps: int = 4) -> dict:
 
 def run_e2e(args, w, run, dev, stream, world: int):
     """The same metric through the host-state API: x, both message buffers and
-    the counters live in pinned host memory and every step streams them
-    through the GPU (HostRelayRun), copies inside the timed region."""
+    the counters live in pinned host memory, and every step is one
+    relay_step_host call that streams them through the GPU (HostRelayRun),
+    copies inside the timed region.  The headline copies every row of m^t
+    back (the step's whole result, as relay_step writes it); `state_only`
+    copies back only the rows a later step reads."""
     import torch
 
     from paper_2110_04175_gb300.host_stream import HostRelayRun
@@ -624,9 +712,8 @@ def run_e2e(args, w, run, dev, stream, world: int):
 
     def pow2(b):  # the pinned allocator rounds every block up to a power of two
         return 1 << max(0, int(b - 1).bit_length())
-    cw = 1 << 22
-    nch = (w.d + cw - 1) // cw
-    need = pow2(nch * w.n * cw * 4) + 2 * pow2(nch * E * cw * 4)
+    ld = (w.d + 31) // 32 * 32
+    need = pow2(w.n * ld * 4) + 2 * pow2(E * ld * 4)
     # every rank on this node pins its own state: split the host's memory
     local_world = max(1, int(os.environ.get("LOCAL_WORLD_SIZE", str(world))))
     avail = host_mem_available()
@@ -640,23 +727,34 @@ def run_e2e(args, w, run, dev, stream, world: int):
     run.x = run.mu = None
     torch.cuda.empty_cache()
     link = host_link_gbs(dev)
+    cw = 1 << 22
     host = HostRelayRun(w.n, w.d, w.edges, chunk=cw, device=dev, mode=w.mode,
-                        c0=shard_offset(int(os.environ.get("RANK", "0")), w.d),
-                        copy_streams=args.copy_streams)
+                        c0=shard_offset(int(os.environ.get("RANK", "0")), w.d), full_output=True)
     host.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
-    host.step(w.lr, w.seed)  # warm-up
-    host.sync()
-    barrier(world)
-    t0 = time.perf_counter()
-    for _ in range(args.e2e_steps):
-        host.step(w.lr, w.seed)
-    host.sync()
-    ms = reduce_max((time.perf_counter() - t0) * 1e3, world)
-    h2d, d2h = host.bytes_per_step()
+
+    def timed(steps: int):
+        host.step(w.lr, w.seed)  # warm-up
+        host.sync()
+        barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            host.step(w.lr, w.seed)
+        host.sync()
+        ms = reduce_max((time.perf_counter() - t0) * 1e3, world)
+        h2d, d2h = host.bytes_per_step()
+        return {"value": round(world * steps / (ms / 1e3), 4), "unit": "steps/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": steps,
+                "copy_gbs": round((h2d + d2h) * steps / (ms / 1e3) / 1e9, 1),
+                "copy_frac": round((h2d + d2h) * steps / (ms / 1e3) / 1e9 / link["both_gbs"], 3)}
+
+    full = timed(args.e2e_steps)
+    host.set_full_output(False)
+    state_only = timed(args.e2e_steps)
+    state_only["note"] = "only the message rows a later step reads come back (not those arriving at leaves)"
     fused = None
     if args.fused_steps > 0:
-        # the same host-state path with relay_steps: the state crosses the
-        # link once per call of K steps (one relay_steps call per chunk visit)
+        # the same host-state path with relay_steps_host: the state crosses
+        # the link once per call of K steps (one relay_steps call per chunk)
         K = args.fused_steps
         host.steps(2, w.lr, w.seed)
         host.sync()
@@ -665,19 +763,16 @@ def run_e2e(args, w, run, dev, stream, world: int):
         host.steps(K, w.lr, w.seed)
         host.sync()
         fms = reduce_max((time.perf_counter() - t1) * 1e3, world)
+        h2d, d2h = host.bytes_per_step()
         fused = {"value": round(world * K / (fms / 1e3), 4), "unit": "steps/s", "steps_per_call": K,
                  "h2d_bytes_per_call": h2d, "d2h_bytes_per_call": d2h,
-                 "note": "HostRelayRun.steps: one relay_steps call per chunk visit"}
-    return {"value": round(world * args.e2e_steps / (ms / 1e3), 4), "unit": "steps/s",
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
-            "path": "HostRelayRun: state in pinned host memory, streamed through the GPU in "
-                    f"{host.nchunks} chunks of {cw} coordinates ({args.copy_streams} copy-in / "
-                    f"kernel / {args.copy_streams} copy-out streams), copies inside the timed region; "
-                    "x, the counters and the message rows a later step reads cross the link",
-            "copy_gbs": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9, 1),
-            "host_link": link,
-            "copy_frac": round((h2d + d2h) * args.e2e_steps / (ms / 1e3) / 1e9 / link["both_gbs"], 3),
-            "fused_steps": fused}
+                 "note": "relay_steps_host: one relay_steps call per chunk visit"}
+    return {**full,
+            "path": "relay_step_host (C ABI): state in pinned host memory in the device layout, streamed "
+                    f"through the GPU in {host.nchunks} chunks of {cw} coordinates (copy-in / kernel / "
+                    "copy-out streams of the library's plan), copies inside the timed region; x and the "
+                    "counters both ways, the message rows the step reads in, every row of m^t out",
+            "host_link": link, "state_only": state_only, "fused_steps": fused}
 
 
 def traffic_per_launch(w, objective: str, kernel: str = "relay_models_kernel", optimizer: str = "sgd"):
@@ -706,8 +801,6 @@ def main(argv=None):
     p.add_argument("--impl", choices=["native", "reference"], default="native")
     p.add_argument("--workload", default=DEFAULT_WORKLOAD)
     p.add_argument("--e2e-steps", type=int, default=5)
-    p.add_argument("--copy-streams", type=int, default=2,
-                   help="copy streams per direction of the host-state path")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--kernel", choices=["auto", "walk", "nodes"], default="auto",
                    help="step kernel (relay_set_kernel)")
@@ -727,6 +820,8 @@ def main(argv=None):
     p.add_argument("--fused-steps", type=int, default=64,
                    help="also time relay_steps with this many steps per call (0: skip); reported "
                         "under 'fused_steps', beside the per-step headline")
+    p.add_argument("--no-per-workload", dest="per_workload", action="store_false",
+                   help="skip the other HBM-bound workloads (reported under 'per_workload')")
     p.add_argument("--d", type=int, default=None,
                    help="override the workload's d (small cases for profiling; not a bench line)")
     args = p.parse_args(argv)

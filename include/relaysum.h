@@ -19,7 +19,8 @@
  *
  * Conventions shared by every call:
  *   - Layout.  x and mu are fp32 [n][ld], messages fp32 [E][ld] with
- *     E = 2(n-1), counters int32 [E]; ld = relay_ld(h) >= d is the padded
+ *     E = 2(n-1) (more rows with received sums: relay_message_rows),
+ *     counters int32 [E]; ld = relay_ld(h) >= d is the padded
  *     row stride (a multiple of 32 floats; relay_set_strides sets others).
  *     The kernels touch columns [0, 4 ceil(d/4)) of each row only; init
  *     zeroes the ragged columns [d, 4 ceil(d/4)), whose values after a step
@@ -154,6 +155,30 @@ int relay_set_kernel(relay_handle *h, int32_t kernel);
  * RELAY_KERNEL_NODES (RELAY_KERNEL_AUTO resolved), or RELAY_EINVAL. */
 int relay_get_kernel(const relay_handle *h);
 
+/* Received sums (an implementation choice; Algorithm 1 fixes only what is
+ * computed).  A worker i with more than 4 neighbours ("wide", such as a
+ * star's hub) sends every neighbour j the message x_i^{t+1/2} + S_i^{t-1} -
+ * m^{t-1}_{j->i}, where S_i^{t-1} = sum_k m^{t-1}_{k->i} is the sum of the
+ * messages it received at step t-1 -- the sum Alg. 1's rebuild line formed
+ * in that step.  With enable = 1 every message buffer carries, after its E
+ * message rows, one row per wide node (in ascending worker id) holding that
+ * sum for the messages in the buffer: relay_step reads S_i^{t-1} from
+ * msg_in's row and writes S_i^t to msg_out's, so each incoming message row
+ * is read once per step instead of twice.  Buffers then have
+ * relay_message_rows(h) rows; relay_init zeroes them all, and msg_in must
+ * be a buffer that relay_init or a relay_step of this handle wrote (or one
+ * whose sum rows the caller keeps equal to the sums of its message rows).
+ * The models and messages agree with the default path within rounding (the
+ * same sums, summed in another order) and the counters are identical.
+ * Rebuilds the handle's visit program (host work only).  Default 0.
+ * Errors: RELAY_EINVAL unless enable is 0 or 1; RELAY_EUNSUPPORTED if the
+ * walk would need more than 127 slots. */
+int relay_set_received_sums(relay_handle *h, int32_t enable);
+
+/* Rows of a message buffer: E, plus one per wide node when received sums
+ * are on (relay_set_received_sums); RELAY_EINVAL for a NULL handle. */
+int32_t relay_message_rows(const relay_handle *h);
+
 /* Absolute index of this handle's first coordinate within a longer model
  * vector (c0 >= 0, a multiple of 4): the noise of local coordinate c is
  * that of coordinate c0 + c, so a vector split into slices -- across GPUs,
@@ -174,6 +199,25 @@ int relay_set_objective(relay_handle *h, const float *mu, float sigma);
  * non-zeros. */
 int relay_set_objective_generated(relay_handle *h, const float *mix, int32_t K, float mu_scale,
                                   uint64_t mu_seed, float sigma);
+
+/* Writes the K Gaussian centres N_1 .. N_K themselves (Philox stream 1, row
+ * k, at the handle's coordinate offset) to `centres`, a device fp32 [K][ld]
+ * array (stride ld_x); the columns [d, 4 ceil(d/4)) are zeroed. */
+int relay_fill_centres(relay_handle *h, float *centres, int32_t K, uint64_t mu_seed, relay_stream_t stream);
+
+/* Binds the same objective with mu formed in the kernel from K stored
+ * Gaussian centres: `centres` is a caller-owned device fp32 [K][ld] array
+ * holding N_1 .. N_K (as relay_fill_centres writes them; read, never
+ * written), `mix` a HOST
+ * fp32 [n][K] matrix whose non-zeros are copied into the handle.  mu_i =
+ * mu_scale * sum_k mix[i][k] N_k is formed in fp32 in the order
+ * relay_fill_objective uses, so every result equals that of the stored mu
+ * bit for bit, while a step reads K centre rows instead of n rows of mu --
+ * fewer bytes when K < n (a mixture of few centres, such as the Dirichlet
+ * mixtures of the heterogeneity experiments).  RELAY_EUNSUPPORTED if K > 16
+ * or mix has more than 1024 non-zeros. */
+int relay_set_objective_centres(relay_handle *h, const float *centres, const float *mix, int32_t K,
+                                float mu_scale, float sigma);
 
 /* Fills mu (device fp32 [n][ld]) with mu_i(c) = mu_scale * sum_k
  * mix[i][k] N_k(c): K Gaussian centres N_k (Philox stream 1, row k) mixed by
@@ -215,6 +259,29 @@ int relay_step(relay_handle *h, float *x, const float *msg_in, float *msg_out,
                int32_t *counts, float lr, uint64_t seed, int64_t step,
                relay_stream_t stream);
 
+/* One RelaySGD iteration t of `count` (1 or 2) handles that split the
+ * coordinates of the same workers into windows -- the double binary trees of
+ * Section 3 ("Spanning trees"): two trees over the n workers, each carrying
+ * half of every model's coordinates, so every worker sends and receives two
+ * half-size messages per step.  The result is that of relay_step(h[k],
+ * x[k], msg_in[k], msg_out[k], counts[k], lr, seed, step, stream) for
+ * k = 0 .. count-1, bit for bit.  When both handles take the walk kernel and
+ * share the objective (the same source; the same mixture when regenerated)
+ * and the local optimiser, their counters are updated by one launch and
+ * their steps by one launch of the step kernel, whose CTAs split between the
+ * windows; otherwise the relay_step calls are issued one after the other.
+ * h, x, msg_in, msg_out, counts: host arrays of `count` entries, each
+ * entry as relay_step takes it (a window's x is usually a column offset
+ * into one model array, with relay_set_strides giving the full row
+ * stride; the caller keeps the windows' columns disjoint).  Errors: those of
+ * relay_step for any window, checked for every window before anything is
+ * enqueued, and RELAY_EINVAL for count outside [1, RELAY_MAX_WINDOWS], a
+ * NULL array or the same handle twice. */
+#define RELAY_MAX_WINDOWS 2
+int relay_step_windows(relay_handle *const *h, int32_t count, float *const *x,
+                       const float *const *msg_in, float *const *msg_out, int32_t *const *counts,
+                       float lr, uint64_t seed, int64_t step, relay_stream_t stream);
+
 /* k consecutive iterations t0, t0+1, ..., t0+k-1 of Algorithm 1 (k >= 0),
  * equal bit for bit to k relay_step calls that alternate the two message
  * buffers: iteration t0+j reads msg_a if j is even (msg_b if odd) and writes
@@ -237,6 +304,84 @@ int relay_step(relay_handle *h, float *x, const float *msg_in, float *msg_out,
 int relay_steps(relay_handle *h, float *x, float *msg_a, float *msg_b, int32_t *counts,
                 float lr, uint64_t seed, int64_t t0, int64_t k, relay_stream_t stream);
 
+/* ---- State in host memory --------------------------------------------
+ *
+ * A state larger than the GPU, or owned by the host, can stay in page-locked
+ * host memory: x [n][ld_x], the message buffers [relay_message_rows][ld_msg]
+ * and the counters [E], in the same layout as on the device (the handle's
+ * strides), allocated with cudaHostAlloc / cudaMallocHost or registered
+ * with cudaHostRegister.  A step streams the coordinates through the GPU in
+ * chunks of `chunk` coordinates: each chunk's x and message rows are copied
+ * in, stepped by the fused kernel at the chunk's absolute coordinate offset,
+ * and copied back, with the copies in both directions and the kernels
+ * overlapped on the plan's own streams.  Every coordinate of Algorithm 1
+ * evolves on its own and the noise is keyed by the absolute coordinate, so
+ * the result equals relay_step on the resident state bit for bit.  The
+ * handle must use regenerated centres (relay_set_objective_generated) and
+ * the SGD local step: a device mu or centres array, or optimiser state, has
+ * no place in a host-state step (RELAY_EUNSUPPORTED otherwise).
+ *
+ * Copies: only the message rows a step reads go in -- every row except
+ * those arriving at a leaf, whose one outgoing message excludes its one
+ * incoming one -- and the same rows come back (the state the next step
+ * needs), unless the plan was created with RELAY_HOST_FULL_OUTPUT, which
+ * copies every row of m^t back, as relay_step writes it.  The rows not
+ * copied back keep whatever the host buffer held.  x and the counters are
+ * copied both ways.  msg_in may equal msg_out: each chunk is read before it
+ * is written, and chunks do not overlap.
+ *
+ * Ordering: a step starts after the work already enqueued on `stream` and
+ * `stream` waits for all of it, so the host arrays may be read after
+ * cudaStreamSynchronize(stream); consecutive steps on the same stream are
+ * ordered.  The plan's streams and events are created by
+ * relay_host_plan_create; relay_step_host and relay_steps_host allocate
+ * nothing and issue one cudaMemcpy2DAsync per array and run of rows per
+ * chunk.  A plan and its staging serve one step at a time. */
+typedef struct relay_host_plan relay_host_plan;
+#define RELAY_HOST_FULL_OUTPUT 1
+
+/* Device staging bytes relay_host_plan_create needs for `buffers` (2..8)
+ * staging sets of one chunk (chunk a positive multiple of 32 coordinates;
+ * capped at d rounded up to 32): (n + 2 rows) * chunk floats per set, plus
+ * the counters.  RELAY_EINVAL for bad arguments. */
+int64_t relay_host_staging_bytes(const relay_handle *h, int64_t chunk, int32_t buffers);
+
+/* Creates a plan for handle h on the current device: `staging` is
+ * caller-owned device memory (256-byte aligned, at least
+ * relay_host_staging_bytes) that the plan uses until destroyed; flags 0 or
+ * RELAY_HOST_FULL_OUTPUT.  Creates three non-blocking streams and the
+ * events that order them.  The plan reads h's settings at every step: keep
+ * h alive while the plan is in use.  Errors: RELAY_EINVAL, RELAY_ENOMEM,
+ * RELAY_ECUDA. */
+int relay_host_plan_create(relay_host_plan **out, relay_handle *h, int64_t chunk, int32_t buffers,
+                           void *staging, int64_t staging_bytes, int32_t flags);
+
+/* Releases the plan's streams and events (NULL allowed); the staging memory
+ * is the caller's. */
+void relay_host_plan_destroy(relay_host_plan *p);
+
+/* Bytes one relay_step_host copies host-to-device and device-to-host. */
+int relay_host_bytes(const relay_host_plan *p, int64_t *h2d, int64_t *d2h);
+
+/* relay_step on a state in host memory (see above): x (in/out), msg_in =
+ * m^{t-1}, msg_out <- m^t, counts c^{t-1} -> c^t, all page-locked host
+ * arrays; lr, seed and step as relay_step.  Errors: RELAY_EINVAL (NULL or
+ * pageable host array, another device than the plan's, step out of range,
+ * no objective), RELAY_EUNSUPPORTED (stored centres or an optimiser with
+ * state), RELAY_ECUDA. */
+int relay_step_host(relay_host_plan *p, float *x, const float *msg_in, float *msg_out, int32_t *counts,
+                    float lr, uint64_t seed, int64_t step, relay_stream_t stream);
+
+/* k steps t0 .. t0+k-1 per chunk visit (relay_steps on each chunk), so the
+ * state crosses the host link once per k steps: x, msg_in = m^{t0-1} and
+ * counts c^{t0-1} go in, x, msg_out <- m^{t0+k-1} and c^{t0+k-1} come back
+ * (the intermediate messages stay on the device).  Every chunk starts from
+ * the same host counters.  The result equals k relay_step_host calls on x,
+ * the counters and m^{t0+k-1}.  RELAY_EUNSUPPORTED for mean estimation
+ * (its counts would advance once per chunk); otherwise as relay_step_host. */
+int relay_steps_host(relay_host_plan *p, float *x, const float *msg_in, float *msg_out, int32_t *counts,
+                     float lr, uint64_t seed, int64_t t0, int64_t k, relay_stream_t stream);
+
 /* The path relay_steps takes on this handle: RELAY_KERNEL_FUSED (several
  * steps per launch), else the per-step kernel of relay_get_kernel; or
  * RELAY_EINVAL. */
@@ -249,9 +394,12 @@ int relay_nbar(const relay_handle *h, const int32_t *counts_host, int32_t *nbar_
 
 /* Introspection of the fused kernel's visit program (for tests and tools):
  * number of shared-memory accumulator slots per thread, the visit order
- * (int32 [n]), per node 10 ints {deg, pos_base, parent_pos, recv_slot,
- * acc_slot, parent_acc, fin_parent, parent, tot_slot, flags} (int32 [n][10];
- * flags bit 0: recv_slot holds the parent's total) and per position 4 ints
+ * (int32 [n]), per node 12 ints {deg, pos_base, parent_pos, recv_slot,
+ * acc_slot, parent_acc, fin_parent, parent, tot_slot, flags, rsum_slot,
+ * rsum_row} (int32 [n][12]; flags bit 0: recv_slot holds the parent's
+ * total; the last two are -1 unless the node is wide and received sums are
+ * on: the slot of its running sum and its sum row, message row
+ * E + rsum_row) and per position 4 ints
  * {in_edge, out_edge, slot, rebuild_in_edge} (int32 [E][4]; the last lists
  * each worker's incoming edges in the order its rebuild adds them); any
  * output pointer may be NULL. */

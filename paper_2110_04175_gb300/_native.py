@@ -26,6 +26,7 @@ RELAY_KERNEL_AUTO = 0
 RELAY_KERNEL_WALK = 1
 RELAY_KERNEL_NODES = 2
 RELAY_KERNEL_FUSED = 3
+RELAY_HOST_FULL_OUTPUT = 1
 
 _lock = threading.Lock()
 _lib = None
@@ -55,6 +56,8 @@ def _load():
             "relay_edges": (ctypes.c_int, [vp, vp, vp]),
             "relay_set_rebuild_mode": (ctypes.c_int, [vp, i32]),
             "relay_set_kernel": (ctypes.c_int, [vp, i32]),
+            "relay_set_received_sums": (ctypes.c_int, [vp, i32]),
+            "relay_message_rows": (i32, [vp]),
             "relay_get_kernel": (ctypes.c_int, [vp]),
             "relay_get_steps_kernel": (ctypes.c_int, [vp]),
             "relay_set_strides": (ctypes.c_int, [vp, i64, i64]),
@@ -64,12 +67,21 @@ def _load():
             "relay_set_coord_offset": (ctypes.c_int, [vp, i64]),
             "relay_set_objective": (ctypes.c_int, [vp, vp, f32]),
             "relay_set_objective_generated": (ctypes.c_int, [vp, vp, i32, f32, u64, f32]),
+            "relay_set_objective_centres": (ctypes.c_int, [vp, vp, vp, i32, f32, f32]),
+            "relay_fill_centres": (ctypes.c_int, [vp, vp, i32, u64, vp]),
             "relay_fill_objective": (ctypes.c_int, [vp, vp, vp, i32, f32, u64, vp]),
             "relay_init": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, vp]),
             "relay_step_counts": (ctypes.c_int, [vp, vp, vp]),
             "relay_step_models": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, vp]),
             "relay_step": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, vp]),
             "relay_steps": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, i64, vp]),
+            "relay_step_windows": (ctypes.c_int, [vp, i32, vp, vp, vp, vp, f32, u64, i64, vp]),
+            "relay_host_staging_bytes": (i64, [vp, i64, i32]),
+            "relay_host_plan_create": (ctypes.c_int, [ctypes.POINTER(vp), vp, i64, i32, vp, i64, i32]),
+            "relay_host_plan_destroy": (None, [vp]),
+            "relay_host_bytes": (ctypes.c_int, [vp, vp, vp]),
+            "relay_step_host": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, vp]),
+            "relay_steps_host": (ctypes.c_int, [vp, vp, vp, vp, vp, f32, u64, i64, i64, vp]),
             "relay_nbar": (ctypes.c_int, [vp, vp, vp]),
             "relay_program": (ctypes.c_int, [vp, vp, vp, vp, vp]),
             "relay_metrics_workspace": (i64, [vp]),
@@ -189,6 +201,16 @@ def relay_set_kernel(h, kernel: int):
     _check(_load().relay_set_kernel(_h(h), int(kernel)), "relay_set_kernel")
 
 
+def relay_set_received_sums(h, enable: bool):
+    _check(_load().relay_set_received_sums(_h(h), int(bool(enable))), "relay_set_received_sums")
+
+
+def relay_message_rows(h) -> int:
+    r = int(_load().relay_message_rows(_h(h)))
+    _check(min(r, 0), "relay_message_rows")
+    return r
+
+
 def relay_get_kernel(h) -> int:
     k = _load().relay_get_kernel(_h(h))
     _check(min(k, 0), "relay_get_kernel")
@@ -244,6 +266,18 @@ def relay_set_objective_generated(h, mix, K: int, mu_scale: float, mu_seed: int,
            "relay_set_objective_generated")
 
 
+def relay_set_objective_centres(h, centres, mix, K: int, mu_scale: float, sigma: float):
+    """centres: device float32 [K][ld] (N_1 .. N_K); mix: host float32 [n][K] (numpy)."""
+    m = np.ascontiguousarray(np.asarray(mix, dtype=np.float32))
+    _check(_load().relay_set_objective_centres(_h(h), _ptr(centres), m.ctypes.data if m.size else None, int(K),
+                                               float(mu_scale), float(sigma)), "relay_set_objective_centres")
+
+
+def relay_fill_centres(h, centres, K: int, mu_seed: int, stream=None):
+    _check(_load().relay_fill_centres(_h(h), _ptr(centres), int(K), int(mu_seed), _stream(stream)),
+           "relay_fill_centres")
+
+
 def relay_fill_objective(h, mu, mix, K: int, mu_scale: float, mu_seed: int, stream=None):
     _check(_load().relay_fill_objective(_h(h), _ptr(mu), _ptr(mix), int(K), float(mu_scale),
                                         int(mu_seed), _stream(stream)), "relay_fill_objective")
@@ -267,6 +301,61 @@ def relay_step_models(h, x, msg_in, msg_out, counts, lr: float, seed: int, step:
 def relay_step(h, x, msg_in, msg_out, counts, lr: float, seed: int, step: int, stream=None):
     _check(_load().relay_step(_h(h), _ptr(x), _ptr(msg_in), _ptr(msg_out), _ptr(counts),
                               float(lr), int(seed), int(step), _stream(stream)), "relay_step")
+
+
+def relay_step_windows(hs, xs, msg_ins, msg_outs, counts, lr: float, seed: int, step: int, stream=None):
+    """relay_step over the tree windows hs[k] (x, messages, counters per window),
+    in one launch of the step kernel where the windows allow it."""
+    k = len(hs)
+    arr = ctypes.c_void_p * max(k, 1)
+    _check(_load().relay_step_windows(arr(*[_h(h) for h in hs]), k, arr(*[_ptr(v) for v in xs]),
+                                      arr(*[_ptr(v) for v in msg_ins]), arr(*[_ptr(v) for v in msg_outs]),
+                                      arr(*[_ptr(v) for v in counts]), float(lr), int(seed), int(step),
+                                      _stream(stream)), "relay_step_windows")
+
+
+class RelayHostPlan:
+    """Owns a relay_host_plan* (and keeps its handle and staging alive)."""
+
+    def __init__(self, raw: int, h, staging):
+        self.raw, self.h, self.staging = raw, h, staging
+        self._lib = _load()
+
+    def __del__(self):
+        if getattr(self, "raw", None):
+            self._lib.relay_host_plan_destroy(self.raw)
+            self.raw = None
+
+
+def relay_host_staging_bytes(h, chunk: int, buffers: int) -> int:
+    r = int(_load().relay_host_staging_bytes(_h(h), int(chunk), int(buffers)))
+    _check(min(r, 0), "relay_host_staging_bytes")
+    return r
+
+
+def relay_host_plan_create(h, chunk: int, buffers: int, staging, flags: int = 0) -> RelayHostPlan:
+    """staging: a device tensor of at least relay_host_staging_bytes bytes."""
+    out = ctypes.c_void_p()
+    _check(_load().relay_host_plan_create(ctypes.byref(out), _h(h), int(chunk), int(buffers), _ptr(staging),
+                                          int(staging.numel() * staging.element_size()), int(flags)),
+           "relay_host_plan_create")
+    return RelayHostPlan(out.value, h, staging)
+
+
+def relay_host_bytes(plan) -> tuple:
+    h2d, d2h = ctypes.c_int64(), ctypes.c_int64()
+    _check(_load().relay_host_bytes(plan.raw, ctypes.addressof(h2d), ctypes.addressof(d2h)), "relay_host_bytes")
+    return int(h2d.value), int(d2h.value)
+
+
+def relay_step_host(plan, x, msg_in, msg_out, counts, lr: float, seed: int, step: int, stream=None):
+    _check(_load().relay_step_host(plan.raw, _ptr(x), _ptr(msg_in), _ptr(msg_out), _ptr(counts), float(lr),
+                                   int(seed), int(step), _stream(stream)), "relay_step_host")
+
+
+def relay_steps_host(plan, x, msg_in, msg_out, counts, lr: float, seed: int, t0: int, k: int, stream=None):
+    _check(_load().relay_steps_host(plan.raw, _ptr(x), _ptr(msg_in), _ptr(msg_out), _ptr(counts), float(lr),
+                                    int(seed), int(t0), int(k), _stream(stream)), "relay_steps_host")
 
 
 def relay_steps(h, x, msg_a, msg_b, counts, lr: float, seed: int, t0: int, k: int, stream=None):
@@ -304,11 +393,11 @@ def relay_nbar(h, counts_host) -> np.ndarray:
 
 
 def relay_program(h):
-    """(nslots, order[n], node_rec[n][10], pos_rec[E][4]) of the step kernels' visit program."""
+    """(nslots, order[n], node_rec[n][12], pos_rec[E][4]) of the step kernels' visit program."""
     n, E = h.n, relay_num_edges(h)
     nslots = ctypes.c_int32()
     order = np.zeros(n, dtype=np.int32)
-    node = np.zeros((n, 10), dtype=np.int32)
+    node = np.zeros((n, 12), dtype=np.int32)
     pos = np.zeros((max(E, 1), 4), dtype=np.int32)
     _check(_load().relay_program(_h(h), ctypes.addressof(nslots), order.ctypes.data,
                                  node.ctypes.data, pos.ctypes.data), "relay_program")
@@ -320,7 +409,8 @@ class _TreeState:
 
     def __init__(self, h, col0: int, d: int, E: int, msg, counts):
         self.h, self.col0, self.d, self.E = h, col0, d, E
-        self.msg = msg          # two [E][ld_msg] buffers (double buffering)
+        self.msg = msg          # two [rows][ld_msg] buffers (double buffering): E messages, then
+                                # the received sums of the wide nodes, if any
         self.counts = counts    # int32 [E]
         self.cur = 0            # msg[cur] holds m^{t-1}
 
@@ -339,22 +429,25 @@ class RelayRun:
     `edges` is one tree, or a list of trees that split the coordinates into
     contiguous quad-aligned windows of the same model array -- the double
     binary trees of Section 3 are a list of two.  Buffers: x [n][ld], per tree
-    two message buffers [E][ld_tree] (double buffering) and counters int32
-    [E], and -- for objective="stored" -- the centres mu [n][ld]
-    (objective="generated" lets the kernel regenerate them).  ``step()``
-    enqueues one relay_step per tree on the current torch stream.
+    two message buffers [rows][ld_tree] (double buffering; rows = E plus the
+    wide nodes' received sums) and counters int32 [E], and -- for
+    objective="stored" -- the centres mu [n][ld] (objective="generated" lets
+    the kernel regenerate them).  ``step()`` enqueues one step on the current
+    torch stream: relay_step, or relay_step_windows for several trees.
     """
 
     def __init__(self, n: int, d: int, edges, device="cuda", mode: int = 1, c0: int = 0,
                  objective: str = "stored", optimizer=None, algorithm: str = "relaysgd",
-                 kernel: str = "auto"):
+                 kernel: str = "auto", received_sums: bool = True):
         """optimizer: None (SGD), ("nesterov", beta1) or ("adam", beta1, beta2, eps);
         algorithm: "relaysgd" (Alg. 1), "grad" (Alg. 6) or "dme" (Alg. 5, x holds
         the running sums y and `dme_count` the counts s of each tree);
-        kernel: "auto", "walk" or "nodes" (relay_set_kernel)."""
+        kernel: "auto", "walk" or "nodes" (relay_set_kernel);
+        received_sums: message buffers carry the wide nodes' received sums
+        (relay_set_received_sums; no effect on trees without a node of degree > 4)."""
         import torch
-        if objective not in ("stored", "generated"):
-            raise ValueError(f"objective must be 'stored' or 'generated', not {objective!r}")
+        if objective not in ("stored", "generated", "centres", "auto"):
+            raise ValueError(f"objective must be 'stored', 'generated', 'centres' or 'auto', not {objective!r}")
         if kernel not in ("auto", "walk", "nodes"):
             raise ValueError(f"kernel must be 'auto', 'walk' or 'nodes', not {kernel!r}")
         trees = list(edges) if isinstance(edges, (list, tuple)) else [edges]
@@ -364,7 +457,7 @@ class RelayRun:
         self.ld = (d + 31) // 32 * 32
         f32 = dict(dtype=torch.float32, device=self.device)
         self.x = torch.empty(n, self.ld, **f32)
-        self.mu = torch.empty(n, self.ld, **f32) if objective == "stored" else None
+        self.mu = None  # stored: [n][ld]; centres: [K][ld], allocated by init() once K is known
         kind = {None: RELAY_OPT_SGD, "nesterov": RELAY_OPT_NESTEROV, "adam": RELAY_OPT_ADAM}[
             optimizer[0] if optimizer else None]
         self.state = [torch.empty(n, self.ld, **f32) for _ in range(kind)]  # m (and v)
@@ -375,6 +468,7 @@ class RelayRun:
             col0 = 4 * q_lo
             dk = min(4 * q_hi, d) - col0 if q_hi > q_lo else 0
             h = relay_create(n, dk, tree_edges)
+            relay_set_received_sums(h, received_sums)
             relay_set_rebuild_mode(h, mode)
             relay_set_kernel(h, {"auto": RELAY_KERNEL_AUTO, "walk": RELAY_KERNEL_WALK,
                                  "nodes": RELAY_KERNEL_NODES}[kernel])
@@ -391,7 +485,8 @@ class RelayRun:
                          if algo == RELAY_ALGO_DME else None)
             relay_set_algorithm(h, algo, dme_count)
             E = relay_num_edges(h)
-            msg = [torch.empty(max(E, 1), max(ld_m, 1), **f32) for _ in range(2)]
+            rows = relay_message_rows(h)  # E, + the wide nodes' received sums
+            msg = [torch.empty(max(rows, 1), max(ld_m, 1), **f32) for _ in range(2)]
             counts = torch.zeros(max(E, 1), dtype=torch.int32, device=self.device)
             tr = _TreeState(h, col0, dk, E, msg, counts)
             tr.dme_count = dme_count
@@ -432,16 +527,29 @@ class RelayRun:
         return _window_ptr(self.x, tr.col0) if tr.d > 0 else None
 
     def init(self, x0_std: float, seed: int, mix, mu_scale: float, mu_seed: int, sigma: float):
+        """objective "stored": mu [n][ld] filled on the device; "centres": the K
+        Gaussian centres [K][ld] stored, mu mixed in the kernel; "generated":
+        nothing stored; "auto": centres when K < n (fewer rows to read),
+        else stored.  All give the same bits."""
         import torch
         mix = np.asarray(mix, dtype=np.float32)
-        mix_t = None
+        K = mix.shape[1]
+        source = self.objective
+        if source == "auto":
+            source = "centres" if 0 < K < self.n and K <= 16 else "stored"
+        self.objective_source = source
+        rows = {"stored": self.n, "centres": K, "generated": 0}[source]
+        if rows and (self.mu is None or self.mu.shape[0] != rows):
+            self.mu = torch.empty(rows, self.ld, dtype=torch.float32, device=self.device)
+        mix_t = torch.as_tensor(mix, device=self.device).contiguous() if source == "stored" else None
         for tr in self.trees:
-            if self.objective == "stored":
-                if mix_t is None:
-                    mix_t = torch.as_tensor(mix, device=self.device).contiguous()
-                mu = _window_ptr(self.mu, tr.col0) if tr.d > 0 else None
-                relay_fill_objective(tr.h, mu, mix_t, mix_t.shape[1], mu_scale, mu_seed)
+            mu = _window_ptr(self.mu, tr.col0) if tr.d > 0 and self.mu is not None else None
+            if source == "stored":
+                relay_fill_objective(tr.h, mu, mix_t, K, mu_scale, mu_seed)
                 relay_set_objective(tr.h, mu, sigma)
+            elif source == "centres":
+                relay_fill_centres(tr.h, mu, K, mu_seed)
+                relay_set_objective_centres(tr.h, mu, mix, K, mu_scale, sigma)
             else:
                 relay_set_objective_generated(tr.h, mix, mix.shape[1], mu_scale, mu_seed, sigma)
             relay_init(tr.h, self._x(tr), tr.msg[0], tr.msg[1], tr.counts, x0_std, seed)
@@ -507,11 +615,11 @@ class RelayRun:
         relay_set_lost_messages(self.trees[tree].h, lost)
 
     def _per_tree(self, issue, stream):
-        """Calls issue(tree, stream) for every tree.  One tree runs on
-        `stream` (default: the current stream).  With several trees (double
-        binary trees) the windows, which share no data, run on streams forked
-        from `stream` and joined back to it, so one window's last wave
-        overlaps the next window's start."""
+        """Calls issue(tree, stream) for every tree (relay_steps).  One tree
+        runs on `stream` (default: the current stream).  With several trees
+        (double binary trees) the windows, which share no data, run on
+        streams forked from `stream` and joined back to it, so one window's
+        last wave overlaps the next window's start."""
         if len(self.trees) == 1:
             issue(self.trees[0], stream)
             return
@@ -537,12 +645,19 @@ class RelayRun:
             main.wait_event(done)
 
     def step(self, lr: float, seed: int, stream=None):
-        """Enqueues one step (relay_step per tree) on `stream`."""
-        def issue(tr, s):
-            relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed, self.t, s)
+        """Enqueues one step on `stream` (default: the current stream): relay_step,
+        or with several tree windows one relay_step_windows call (one counter
+        launch and one step-kernel launch for both windows where they allow it)."""
+        trs = self.trees
+        if len(trs) == 1:
+            tr = trs[0]
+            relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed, self.t, stream)
+        else:
+            relay_step_windows([tr.h for tr in trs], [self._x(tr) for tr in trs], [tr.msg[tr.cur] for tr in trs],
+                               [tr.msg[1 - tr.cur] for tr in trs], [tr.counts for tr in trs], lr, seed, self.t,
+                               stream)
+        for tr in trs:
             tr.cur = 1 - tr.cur
-
-        self._per_tree(issue, stream)
         self.t += 1
 
     def steps(self, k: int, lr: float, seed: int, stream=None):

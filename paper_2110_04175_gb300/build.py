@@ -1,8 +1,9 @@
 """Builds librelaysum.so in-tree with nvcc for sm_103a (GB300).
 
-Two translation units compiled in parallel (host program builder, CUDA
-kernels + C ABI), linked into one shared library with the CUDA runtime
-statically linked, so the library loads on a machine without a GPU.
+Three translation units compiled in parallel (host program builder, CUDA
+kernels + C ABI, host-state step), linked into one shared library with the
+CUDA runtime statically linked, so the library loads on a machine without a
+GPU.
 """
 from __future__ import annotations
 
@@ -18,8 +19,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "librelaysum.so")
 
-SOURCES = ["program.cpp", "relaysum.cu"]
-HEADERS = [os.path.join(CSRC, "program.h"), os.path.join(INCLUDE, "relaysum.h")]
+SOURCES = ["program.cpp", "relaysum.cu", "host_step.cpp"]
+HEADERS = [os.path.join(CSRC, "program.h"), os.path.join(CSRC, "handle.h"), os.path.join(INCLUDE, "relaysum.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
               "-I" + INCLUDE, "-I" + CSRC]

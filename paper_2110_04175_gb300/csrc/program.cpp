@@ -94,7 +94,7 @@ struct Walk {
     std::vector<std::vector<int>> children;
 };
 
-Walk make_walk(const Tree& t, int root) {
+Walk make_walk(const Tree& t, int root, bool received_sums) {
     const int n = t.n;
     Walk w;
     w.parent.assign(n, -1);
@@ -127,7 +127,8 @@ Walk make_walk(const Tree& t, int root) {
         const int D = static_cast<int>(t.nbr[i].size());
         const bool wide = D > kRegDeg;
         const int has_parent = w.parent[i] >= 0 ? 1 : 0;
-        const int own = (m > 0) ? (wide ? 2 : 1) : 0;             // accumulator (+ total)
+        // accumulator (+ total, + received sum)
+        const int own = (m > 0) ? (wide ? (received_sums ? 3 : 2) : 1) : 0;
         vpeak[i] = std::max(has_parent, own + (wide ? 0 : m));     // slots at i's own visit
         std::stable_sort(ch.begin(), ch.end(), [&](int a, int b) { return need[a] > need[b]; });
         auto peak_of = [&](const std::vector<int>& order) {
@@ -175,7 +176,7 @@ Walk make_walk(const Tree& t, int root) {
 
 // Assigns slots along the walk (lowest free id first) and fills the
 // program; returns the number of slots used.
-int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
+int assign_slots(const Tree& t, const Walk& w, int root, bool received_sums, Program* p) {
     const int n = t.n;
     std::priority_queue<int, std::vector<int>, std::greater<int>> free_ids;
     int next_id = 0;
@@ -190,7 +191,7 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
     auto release = [&](int s) {
         if (s >= 0) free_ids.push(s);
     };
-    std::vector<int> recv(n, -1), acc(n, -1), tot(n, -1), pos_base(n, 0);
+    std::vector<int> recv(n, -1), acc(n, -1), tot(n, -1), rsum(n, -1), pos_base(n, 0);
     int base = 0;
     for (int i = 0; i < n; ++i) {
         pos_base[i] = base;
@@ -208,6 +209,8 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
         if (!par_wide) release(recv[i]);
         acc[i] = (m > 0) ? alloc() : -1;
         tot[i] = (wide && m > 0) ? alloc() : -1;
+        rsum[i] = (wide && m > 0 && received_sums) ? alloc() : -1;
+        p->rsum_slot[i] = static_cast<int8_t>(rsum[i]);
         int parent_pos = -1;
         for (int s = 0; s < D; ++s) {
             const int k = t.nbr[i][s];
@@ -241,6 +244,7 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
         if (last) {
             release(acc[par]);
             release(tot[par]);
+            release(rsum[par]);
         }
         p->order[v] = static_cast<int16_t>(i);
     }
@@ -262,27 +266,36 @@ int assign_slots(const Tree& t, const Walk& w, int root, Program* p) {
 
 }  // namespace
 
-int build_program(int n, const int32_t* edges, int n_edges, Program* out) {
+int build_program(int n, const int32_t* edges, int n_edges, Program* out, bool received_sums) {
     std::memset(out, 0, sizeof(Program));
     Tree t;
     const int rc = validate(n, edges, n_edges, &t, out);
     if (rc != RELAY_OK) return rc;
     out->n = n;
     out->E = 2 * (n - 1);
+    // rows of received sums: the wide nodes in ascending id
+    std::memset(out->rsum_row, -1, sizeof(out->rsum_row));
+    std::memset(out->rsum_slot, -1, sizeof(out->rsum_slot));
+    out->nwide = 0;
+    if (received_sums)
+        for (int i = 0; i < n; ++i)
+            if (static_cast<int>(t.nbr[i].size()) > kRegDeg) out->rsum_row[i] = static_cast<int8_t>(out->nwide++);
     int best_root = 0, best_slots = -1;
     Program trial;
     for (int r = 0; r < n; ++r) {
         std::memcpy(&trial, out, sizeof(Program));
-        const Walk w = make_walk(t, r);
-        const int s = assign_slots(t, w, r, &trial);
+        const Walk w = make_walk(t, r, received_sums);
+        const int s = assign_slots(t, w, r, received_sums, &trial);
         if (best_slots < 0 || s < best_slots) {
             best_slots = s;
             best_root = r;
         }
     }
-    const Walk w = make_walk(t, best_root);
-    out->nslots = assign_slots(t, w, best_root, out);
+    const Walk w = make_walk(t, best_root, received_sums);
+    out->nslots = assign_slots(t, w, best_root, received_sums, out);
     out->root = best_root;
+    // a received-sum slot must fit its int8 field
+    if (received_sums && out->nwide > 0 && out->nslots > 127) return RELAY_EUNSUPPORTED;
     return RELAY_OK;
 }
 

@@ -21,6 +21,16 @@
 //     message) and writes it out.  This keeps the slots per thread O(1)
 //     instead of O(degree).
 //
+// Received sums (optional, relay_set_received_sums).  The sum a wide node
+// needs, S_i^{t-1} = sum_k m^{t-1}_{k->i}, is the sum of received messages
+// that Alg. 1's rebuild line formed one step earlier.  With received sums
+// on, every message buffer carries one more row per wide node holding it:
+// the walk forms T_i = x_i^{t+1/2} + S_i^{t-1} from that one row instead of
+// reading all D incoming rows, each child's m^{t-1}_{c->i} is then read
+// once (at the child's visit) rather than twice, and S_i^t is summed in one
+// more slot (rsum_slot) as the new messages arrive and written to row
+// E + rsum_row[i] of the output buffer at the visit of i's last child.
+//
 // The same program drives the node-parallel kernel for short vectors (one
 // thread per worker and quad): it forms each worker's messages with the
 // walk's arithmetic and adds the incoming ones in the walk's order (rb_in),
@@ -68,6 +78,13 @@ struct Program {
     int16_t rb_in[kMaxE];        // i's positions: its incoming edges in the walk's rebuild
                                  // order (from the DFS parent, then from the children in
                                  // visit order); the node-parallel kernel adds them so
+    // received sums (built only when they are on; else -1): a wide node's
+    // slot of its running sum S_i^t, and its row among the sum rows (row
+    // E + rsum_row[i] of a message buffer).  int8 keeps two programs within
+    // one launch's parameter space.
+    int8_t rsum_slot[kMaxN];
+    int8_t rsum_row[kMaxN];
+    int32_t nwide;               // rows of received sums (0 when they are off)
 };
 
 // Where the kernel takes the quadratic centres mu_i from.
@@ -78,6 +95,7 @@ enum ObjectiveSource : int32_t {
     kMuStored = 0,      // read the caller's mu array
     kMuPerRow = 1,      // regenerate: one Philox block per non-zero weight of the row
     kMuCachedCentres = 2,  // regenerate the K centres once per quad, then mix per row
+    kMuStoredCentres = 3,  // read the caller's K centres once per quad, then mix per row
 };
 
 struct Objective {
@@ -90,7 +108,8 @@ struct Objective {
     float w[kMaxMixNnz];          // weight
 };
 
-// Status codes mirror relaysum.h.
-int build_program(int n, const int32_t* edges, int n_edges, Program* out);
+// Status codes mirror relaysum.h.  received_sums: lay out the walk for
+// received-sum rows (one more slot per wide node).
+int build_program(int n, const int32_t* edges, int n_edges, Program* out, bool received_sums = false);
 
 }  // namespace relaysum

@@ -35,6 +35,7 @@
 #include <cstring>
 #include <new>
 
+#include "handle.h"
 #include "program.h"
 #include "relaysum.h"
 
@@ -45,29 +46,6 @@ using relaysum::NodeRec;
 using relaysum::Objective;
 using relaysum::Program;
 
-struct relay_handle {
-    Program prog;
-    Objective obj;
-    int64_t d = 0, ld = 0, nquads = 0, c0 = 0;
-    int64_t ld_x = 0, ld_m = 0;  // row strides (floats) of x / mu and of the messages
-    int32_t mode = 1;
-    const float* mu = nullptr;
-    float sigma = 0.0f;
-    bool has_objective = false;
-    // local optimiser of Alg. 1's local step (appendix "RelaySGD with momentum / Adam")
-    int32_t opt = 0;
-    float beta1 = 0.0f, beta2 = 0.0f, eps = 0.0f;
-    float* s1 = nullptr;  // momentum buffer / Adam first moment, [n][ld_x]
-    float* s2 = nullptr;  // Adam second moment, [n][ld_x]
-    // algorithm on the relay: 0 RelaySGD (Alg. 1), 1 RelaySum/Grad (Alg. 6), 2 DME (Alg. 5)
-    int32_t algo = 0;
-    int64_t* dme_count = nullptr;  // algo 2: s_i, device int64 [n]
-    // step kernel: RELAY_KERNEL_AUTO / _WALK / _NODES
-    int32_t kernel = RELAY_KERNEL_AUTO;
-    // messages lost in transit (Section 4.4), one bit per directed edge
-    bool has_lost = false;
-    uint32_t lost[relaysum::kMaxE / 32 + 1] = {};
-};
 
 namespace {
 
@@ -213,10 +191,27 @@ __device__ __forceinline__ int32_t next_count(const Program& prog, const LostMas
     return (has_lost && lost(e)) ? 0 : s;
 }
 
-__global__ void relay_counts_kernel(const __grid_constant__ Program prog, const __grid_constant__ LostMask lost,
-                                    int has_lost, int32_t* counts, int64_t* dme_count) {
+// The counters of NT handles (the tree windows of relay_step_windows, or one
+// handle): CTA w updates window w's.
+template <int NT>
+struct CountWindows {
+    Program prog[NT];
+    LostMask lost[NT];
+    int32_t has_lost[NT];
+    int32_t* counts[NT];
+    int64_t* dme_count[NT];  // Alg. 5's counts s_i, or null
+};
+
+template <int NT>
+__global__ void relay_counts_kernel(const __grid_constant__ CountWindows<NT> cw) {
     allow_dependent_launch();
     __shared__ int32_t c_old[kMaxE];
+    const int w = (NT == 1) ? 0 : static_cast<int>(blockIdx.x);
+    const Program& prog = cw.prog[w];
+    const LostMask& lost = cw.lost[w];
+    const int has_lost = cw.has_lost[w];
+    int32_t* const counts = cw.counts[w];
+    int64_t* const dme_count = cw.dme_count[w];
     const int E = prog.E;
     for (int e = threadIdx.x; e < E; e += blockDim.x) c_old[e] = counts[e];
     __syncthreads();
@@ -233,9 +228,14 @@ __global__ void relay_counts_kernel(const __grid_constant__ Program prog, const 
 }
 
 // The counters (and the mean-estimation counts) advanced by k steps, for
-// relay_steps: one CTA of blockDim >= n threads, the counters of the two
-// step parities in shared memory, one barrier per step.
-__global__ void relay_counts_steps_kernel(const __grid_constant__ Program prog,
+// relay_steps: one CTA of kCountsThreads >= n threads (thread i carries
+// worker i's mean-estimation count), the counters of the two step parities
+// in shared memory, one barrier per step.
+constexpr int kCountsThreads = 256;
+static_assert(kMaxN <= kCountsThreads, "relay_counts_steps_kernel gives each worker its own thread");
+
+__global__ void __launch_bounds__(kCountsThreads)
+relay_counts_steps_kernel(const __grid_constant__ Program prog,
                                           const __grid_constant__ LostMask lost, int has_lost, int32_t* counts,
                                           int64_t* dme_count, int k) {
     __shared__ int32_t c[2][kMaxE];
@@ -276,6 +276,7 @@ struct ModelArgs {
     int mode;         // 0: Alg. 1 rebuild, 1: robust rebuild
     int algo;         // 0 RelaySGD, 1 RelaySum/Grad, 2 mean estimation
     int has_lost;     // any bit of `lost` set
+    int rsum;         // wide nodes read and write their received-sum rows (program.h)
     LostMask lost;    // messages lost in transit this step
     float* s1;        // optimiser state (momentum / Adam m), [n][ld_x]
     float* s2;        // Adam v, [n][ld_x]
@@ -298,21 +299,37 @@ struct Slots {
     __device__ __forceinline__ float4& operator[](int s) const { return base[s * stride]; }
 };
 
-// The message to the DFS parent joins the parent's accumulator; if this
-// worker is the parent's last child, the parent's rebuild is complete.
-__device__ __forceinline__ void to_parent(const NodeRec& r, const ModelArgs& a, int64_t q, float4 out,
-                                          const Slots& sl, const float* s_scale) {
+// Row of wide node i's received sum in a message buffer (program.h).
+__device__ __forceinline__ int64_t rsum_row(const Program& prog, int i) { return prog.E + prog.rsum_row[i]; }
+
+// The message to the DFS parent joins the parent's accumulator (and, with
+// received sums, a wide parent's running sum S_p^t); if this worker is the
+// parent's last child, the parent's rebuild (and S_p^t) is complete.  WIDE:
+// the tree has a node of degree > kRegDeg (the walk's wide-node paths are
+// compiled only then).
+template <bool WIDE>
+__device__ __forceinline__ void to_parent(const Program& prog, const NodeRec& r, const ModelArgs& a, int64_t q,
+                                          float4 out, const Slots& sl, const float* s_scale) {
     const float4 acc = add4(sl[r.parent_acc], out);
     if (r.fin_parent >= 0) {
         st_stream(a.x + r.fin_parent * a.ld_x + 4 * q, scale4(acc, s_scale[r.fin_parent]));
     } else {
         sl[r.parent_acc] = acc;
     }
+    if (WIDE && a.rsum && (r.flags & relaysum::kRecvFromTotal)) {
+        const int rs = prog.rsum_slot[r.parent];
+        const float4 sum = add4(sl[rs], out);
+        if (r.fin_parent >= 0) {
+            st_stream(a.msg_out + rsum_row(prog, r.parent) * a.ld_m + 4 * q, sum);
+        } else {
+            sl[rs] = sum;
+        }
+    }
 }
 
 // Degree D <= kRegDeg: the D incoming messages live in registers; outgoing
 // message s is prefix(s) + suffix(s+1) with prefix(s) = xh + m_0 + ... + m_{s-1}.
-template <int D>
+template <int D, bool WIDE>
 __device__ __forceinline__ void visit_small(const Program& prog, const NodeRec& r, const ModelArgs& a,
                                             int64_t q, float4 xh, const Slots& sl,
                                             const float* s_scale) {
@@ -333,36 +350,43 @@ __device__ __forceinline__ void visit_small(const Program& prog, const NodeRec& 
         const float4 out = delivered(a, e, (s == D - 1) ? pre[s] : add4(pre[s], suf[s + 1]));
         st_stream(a.msg_out + e * a.ld_m + 4 * q, out);
         if (s == r.parent_pos) {
-            to_parent(r, a, q, out, sl, s_scale);
+            to_parent<WIDE>(prog, r, a, q, out, sl, s_scale);
         } else {
             sl[prog.pos_slot[r.pos_base + s]] = out;
         }
     }
 }
 
-// Degree D > kRegDeg: one streaming pass forms T = xh + sum of all incoming
-// messages; the message to the parent is T minus the parent's incoming
-// message, and T stays in a slot for the children (see program.h).  The
-// pass runs over descending positions while the children are visited in
-// ascending order, so the first children re-read the most recently read
-// (L2-resident) rows.
-__device__ __noinline__ void visit_wide(const Program& prog, const NodeRec& r, const ModelArgs& a,
+// Degree D > kRegDeg: T = xh + the sum of all incoming messages; the message
+// to the parent is T minus the parent's incoming message, and T stays in a
+// slot for the children (see program.h).  Without received sums one
+// streaming pass reads the D incoming rows, over descending positions while
+// the children are visited in ascending order, so the first children
+// re-read the most recently read (L2-resident) rows.  With received sums,
+// T = xh + S_i^{t-1} from the one sum row, and only the parent's incoming
+// row is read here.
+__device__ __noinline__ void visit_wide(const Program& prog, const NodeRec& r, const ModelArgs& a, int i,
                                         int64_t q, float4 xh, const Slots& sl,
                                         const float* s_scale) {
     const int D = r.deg;
     const int base = r.pos_base;
     float4 total = xh;
     float4 from_parent = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s = D - 1; s >= 0; --s) {
-        const float4 m = ld_keep(a.msg_in + prog.pos_in[base + s] * a.ld_m + 4 * q);
-        total = add4(total, m);
-        if (s == r.parent_pos) from_parent = m;
+    if (a.rsum) {
+        total = add4(xh, ld_stream(a.msg_in + rsum_row(prog, i) * a.ld_m + 4 * q));
+        if (r.parent_pos >= 0) from_parent = ld_stream(a.msg_in + prog.pos_in[base + r.parent_pos] * a.ld_m + 4 * q);
+    } else {
+        for (int s = D - 1; s >= 0; --s) {
+            const float4 m = ld_keep(a.msg_in + prog.pos_in[base + s] * a.ld_m + 4 * q);
+            total = add4(total, m);
+            if (s == r.parent_pos) from_parent = m;
+        }
     }
     if (r.parent_pos >= 0) {
         const int e = prog.pos_out[base + r.parent_pos];
         const float4 out = delivered(a, e, sub4(total, from_parent));
         st_stream(a.msg_out + e * a.ld_m + 4 * q, out);
-        to_parent(r, a, q, out, sl, s_scale);
+        to_parent<true>(prog, r, a, q, out, sl, s_scale);
     }
     sl[r.tot_slot] = total;
 }
@@ -408,18 +432,26 @@ __device__ __forceinline__ float4 local_update(const ModelArgs& a, int i, int64_
     return u;
 }
 
-// mu_i for quad q: read, or regenerated exactly as relay_fill_mu_kernel
-// writes it (same normals, same fma order), so both sources give the same bits.
+// mu_i for quad q: read, or formed from the K Gaussian centres exactly as
+// relay_fill_mu_kernel writes it (the same normals, the same fma order), so
+// every source gives the same bits.  The centres are regenerated
+// (kMuPerRow, kMuCachedCentres) or read from the caller's [K][ld_x] array
+// (kMuStoredCentres, a.mu); `cen` holds the quad's K centres in shared
+// memory where the walk cached them, else null.
 template <int OBJ>
 __device__ __forceinline__ float4 centre(const Objective& obj, const PhiloxKey& mu_key, const ModelArgs& a,
                                          int i, int64_t q, const float4* cen, int cen_stride) {
     if (OBJ == relaysum::kMuStored) return ld_stream(a.mu + i * a.ld_x + 4 * q);
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int j = obj.row_off[i]; j < obj.row_off[i + 1]; ++j) {
-        const float4 z = (OBJ == relaysum::kMuPerRow)
-                             ? normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(obj.col[j]),
-                                       0u, 1u, mu_key)
-                             : cen[obj.col[j] * cen_stride];
+        float4 z;
+        if (OBJ == relaysum::kMuPerRow) {
+            z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(obj.col[j]), 0u, 1u, mu_key);
+        } else if (OBJ == relaysum::kMuStoredCentres && cen == nullptr) {
+            z = ld_stream(a.mu + obj.col[j] * a.ld_x + 4 * q);
+        } else {
+            z = cen[obj.col[j] * cen_stride];
+        }
         acc = fma4(obj.w[j], z, acc);
     }
     return scale4_rn(acc, obj.scale);
@@ -478,28 +510,49 @@ __device__ __forceinline__ float4 relayed_value(const ModelArgs& a, int i, int64
     return relayed_with(a, xv, mv, z, [&](float4 g) { return local_update<OPT>(a, i, q, g); });
 }
 
+// The step of NT handles in one launch: one handle, or the tree windows of
+// relay_step_windows (the double binary trees of Section 3: two trees over
+// the same workers, each carrying its own columns of the models).  The
+// grid's first `split` CTAs work on window 0, the rest on window 1.
+template <int NT>
+struct Windows {
+    Program prog[NT];
+    ModelArgs a[NT];
+    int32_t split;
+};
+
 // OBJ: where mu comes from (ObjectiveSource).  OPT: the local optimiser
-// (0 SGD, 1 Nesterov momentum, 2 Adam).
-template <int OBJ, int OPT>
+// (0 SGD, 1 Nesterov momentum, 2 Adam).  NT: windows per launch.  WIDE: some
+// node has more than kRegDeg neighbours; without one the wide-node paths are
+// not compiled, and they cost the narrow trees nothing.
+template <int OBJ, int OPT, int NT, bool WIDE>
 __global__ void __launch_bounds__(128)
-relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant__ Objective obj,
-                    const __grid_constant__ PhiloxKey mu_key, const __grid_constant__ ModelArgs a) {
+relay_models_kernel(const __grid_constant__ Windows<NT> win, const __grid_constant__ Objective obj,
+                    const __grid_constant__ PhiloxKey mu_key) {
     extern __shared__ float4 slot_mem[];
     __shared__ float s_scale[kMaxN];
     __shared__ float s_fill[kMaxN];
+    const int wdw = (NT == 1) ? 0 : (static_cast<int>(blockIdx.x) >= win.split ? 1 : 0);
+    const Program& prog = win.prog[wdw];
+    const ModelArgs& a = win.a[wdw];
+    const int64_t cta = (NT == 1) ? blockIdx.x : static_cast<int64_t>(blockIdx.x) - (wdw ? win.split : 0);
+    const int64_t ctas = (NT == 1) ? gridDim.x : (wdw ? static_cast<int64_t>(gridDim.x) - win.split : win.split);
     const int n = prog.n;
     wait_for_prior_grid();
     rebuild_factors(prog, a, s_scale, s_fill);
     __syncthreads();
     const Slots sl{slot_mem + threadIdx.x, static_cast<int>(blockDim.x)};
-    float4* cen = slot_mem + prog.nslots * blockDim.x + threadIdx.x;  // OBJ == kMuCachedCentres
-    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < a.nquads;
-         q += stride) {
+    // the quad's K centres, regenerated or read once per quad (kMuCachedCentres, kMuStoredCentres)
+    float4* cen = slot_mem + prog.nslots * blockDim.x + threadIdx.x;
+    const int64_t stride = ctas * blockDim.x;
+    for (int64_t q = cta * blockDim.x + threadIdx.x; q < a.nquads; q += stride) {
         if (OBJ == relaysum::kMuCachedCentres) {
             for (int k = 0; k < obj.K; ++k)
                 cen[k * blockDim.x] = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k), 0u,
                                               1u, mu_key);
+        }
+        if (OBJ == relaysum::kMuStoredCentres) {
+            for (int k = 0; k < obj.K; ++k) cen[k * blockDim.x] = ld_stream(a.mu + k * a.ld_x + 4 * q);
         }
         // x (and a stored mu) of the next node in the walk are loaded one visit
         // early, so their latency overlaps the current visit's arithmetic
@@ -517,6 +570,15 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
                 xn = *reinterpret_cast<const float4*>(a.x + inext * a.ld_x + 4 * q);
                 if (OBJ == relaysum::kMuStored) mn = ld_stream(a.mu + inext * a.ld_x + 4 * q);
             }
+            // a child of a wide node p forms its incoming message as
+            // T_p - m^{t-1}_{i->p}; that row is loaded before the noise
+            // arithmetic, whose latency it then overlaps (with received sums
+            // this is the one read of m^{t-1}_{i->p})
+            float4 back = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (WIDE && (r.flags & relaysum::kRecvFromTotal)) {
+                const float* mp = a.msg_in + prog.pos_out[r.pos_base + r.parent_pos] * a.ld_m + 4 * q;
+                back = a.rsum ? ld_stream(mp) : __ldg(reinterpret_cast<const float4*>(mp));
+            }
             const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i),
                                      a.step, 0u, a.key);
             const float4 xh = relayed_value<OPT>(a, i, q, xv, mv, z);
@@ -524,25 +586,27 @@ relay_models_kernel(const __grid_constant__ Program prog, const __grid_constant_
             // Alg. 6: n; Alg. 5: 1; Alg. 1: nothing)
             float4 acc = xh;
             if (s_fill[i] != 0.0f) acc = add4(scale4(xv, s_fill[i]), xh);
+            float4 recv = make_float4(0.f, 0.f, 0.f, 0.f);
             if (r.recv_slot >= 0) {
-                float4 recv = sl[r.recv_slot];
-                if (r.flags & relaysum::kRecvFromTotal) {
-                    // m^t_{p->i} = T_p - m^{t-1}_{i->p}, written out here
-                    const int pos = r.pos_base + r.parent_pos;
-                    const int e = prog.pos_in[pos];
-                    recv = delivered(a, e, sub4(recv, __ldg(reinterpret_cast<const float4*>(
-                                                          a.msg_in + prog.pos_out[pos] * a.ld_m + 4 * q))));
+                recv = sl[r.recv_slot];
+                if (WIDE && (r.flags & relaysum::kRecvFromTotal)) {  // m^t_{p->i} = T_p - m^{t-1}_{i->p}, written out here
+                    const int e = prog.pos_in[r.pos_base + r.parent_pos];
+                    recv = delivered(a, e, sub4(recv, back));
                     st_stream(a.msg_out + e * a.ld_m + 4 * q, recv);
                 }
                 acc = add4(acc, recv);
             }
+            // a wide node's received sum S_i^t starts with its DFS parent's message
+            if (WIDE && a.rsum && r.deg > kRegDeg) sl[prog.rsum_slot[i]] = add4(make_float4(0.f, 0.f, 0.f, 0.f), recv);
             switch (r.deg) {
                 case 0: break;
-                case 1: visit_small<1>(prog, r, a, q, xh, sl, s_scale); break;
-                case 2: visit_small<2>(prog, r, a, q, xh, sl, s_scale); break;
-                case 3: visit_small<3>(prog, r, a, q, xh, sl, s_scale); break;
-                case 4: visit_small<4>(prog, r, a, q, xh, sl, s_scale); break;
-                default: visit_wide(prog, r, a, q, xh, sl, s_scale); break;
+                case 1: visit_small<1, WIDE>(prog, r, a, q, xh, sl, s_scale); break;
+                case 2: visit_small<2, WIDE>(prog, r, a, q, xh, sl, s_scale); break;
+                case 3: visit_small<3, WIDE>(prog, r, a, q, xh, sl, s_scale); break;
+                case 4: visit_small<4, WIDE>(prog, r, a, q, xh, sl, s_scale); break;
+                default:
+                    if (WIDE) visit_wide(prog, r, a, i, q, xh, sl, s_scale);
+                    break;
             }
             if (r.acc_slot < 0) {
                 st_stream(a.x + i * a.ld_x + 4 * q, scale4(acc, s_scale[i]));
@@ -592,18 +656,20 @@ __device__ __forceinline__ void node_small(const Program& prog, const NodeRec& r
 }
 
 // Degree D > kRegDeg: T = x^{t+1/2} + the incoming messages summed over
-// descending positions, then message s = T - (incoming message s), as in
-// visit_wide and at the wide node's children.  The incoming messages wait
-// in shared memory (rows of worker i's own incoming edges).
-__device__ __noinline__ void node_wide(const Program& prog, const NodeRec& r, const ModelArgs& a, int64_t q,
-                                       float4 xh, float4* m_new, float4* m_old, int qb) {
+// descending positions (with received sums: + the sum row S_i^{t-1}), then
+// message s = T - (incoming message s), as in visit_wide and at the wide
+// node's children.  The incoming messages wait in shared memory (rows of
+// worker i's own incoming edges).
+__device__ __noinline__ void node_wide(const Program& prog, const NodeRec& r, const ModelArgs& a, int i,
+                                       int64_t q, float4 xh, float4* m_new, float4* m_old, int qb) {
     const int D = r.deg;
     const int base = r.pos_base;
     float4 total = xh;
+    if (a.rsum) total = add4(xh, ld_stream(a.msg_in + rsum_row(prog, i) * a.ld_m + 4 * q));
     for (int s = D - 1; s >= 0; --s) {
         const int ein = prog.pos_in[base + s];
         const float4 m = ld_stream(a.msg_in + ein * a.ld_m + 4 * q);
-        total = add4(total, m);
+        if (!a.rsum) total = add4(total, m);
         m_old[ein * qb] = m;
     }
     for (int s = 0; s < D; ++s) {
@@ -628,8 +694,9 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
     __shared__ float s_scale[kMaxN];
     __shared__ float s_fill[kMaxN];
     // regenerated centres are formed per row (the walk's cached centres are
-    // the same normals mixed in the same order)
-    constexpr int kObj = (OBJ == relaysum::kMuStored) ? relaysum::kMuStored : relaysum::kMuPerRow;
+    // the same normals mixed in the same order); stored centres are read per
+    // non-zero of the row
+    constexpr int kObj = (OBJ == relaysum::kMuCachedCentres) ? relaysum::kMuPerRow : OBJ;
     const int i = static_cast<int>(threadIdx.x) / qb;
     const int qi = static_cast<int>(threadIdx.x) - i * qb;
     float4* const buf0 = node_mem + qi;                     // [e * qb]: m^t on edge e (even blocks)
@@ -675,12 +742,22 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
                 case 2: node_small<2>(prog, r, a, q, xh, m_new, qb); break;
                 case 3: node_small<3>(prog, r, a, q, xh, m_new, qb); break;
                 case 4: node_small<4>(prog, r, a, q, xh, m_new, qb); break;
-                default: node_wide(prog, r, a, q, xh, m_new, m_old, qb); break;
+                default: node_wide(prog, r, a, i, q, xh, m_new, m_old, qb); break;
             }
         }
         __syncthreads();
         if (active) {
-            for (int k = 0; k < r.deg; ++k) acc = add4(acc, m_new[prog.rb_in[r.pos_base + k] * qb]);
+            if (a.rsum && r.deg > kRegDeg) {  // and the wide node's received sum S_i^t, in the same order
+                float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int k = 0; k < r.deg; ++k) {
+                    const float4 m = m_new[prog.rb_in[r.pos_base + k] * qb];
+                    acc = add4(acc, m);
+                    sum = add4(sum, m);
+                }
+                st_stream(a.msg_out + rsum_row(prog, i) * a.ld_m + 4 * q, sum);
+            } else {
+                for (int k = 0; k < r.deg; ++k) acc = add4(acc, m_new[prog.rb_in[r.pos_base + k] * qb]);
+            }
             st_stream(a.x + i * a.ld_x + 4 * q, scale4(acc, s_scale[i]));
         }
     }
@@ -774,7 +851,7 @@ relay_fused_steps_kernel(const __grid_constant__ Program prog, const __grid_cons
                          const __grid_constant__ FusedSteps fs, int qb) {
     extern __shared__ float4 fused_mem[];
     __shared__ int32_t c_mem[2][kMaxE];  // counters of the step parities
-    constexpr int kObj = (OBJ == relaysum::kMuStored) ? relaysum::kMuStored : relaysum::kMuPerRow;
+    constexpr int kObj = (OBJ == relaysum::kMuCachedCentres) ? relaysum::kMuPerRow : OBJ;
     const int tid = static_cast<int>(threadIdx.x);
     const int i = tid / qb;
     const int qi = tid - i * qb;
@@ -870,7 +947,8 @@ relay_fused_steps_kernel(const __grid_constant__ Program prog, const __grid_cons
 
 // --------------------------------------------------------------------- init
 
-__global__ void relay_init_kernel(float* x, float* msg_a, float* msg_b, int n, int E, int64_t ld_x,
+// rows: message rows to zero (E, plus the received-sum rows when they are on).
+__global__ void relay_init_kernel(float* x, float* msg_a, float* msg_b, int n, int rows, int64_t ld_x,
                                   int64_t ld_m, int64_t nquads, int64_t d, uint32_t q0, float x0_std,
                                   const __grid_constant__ PhiloxKey key) {
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -881,7 +959,7 @@ __global__ void relay_init_kernel(float* x, float* msg_a, float* msg_b, int n, i
                                      c + 2 < d ? x0_std * z.z : 0.f, c + 3 < d ? x0_std * z.w : 0.f);
         for (int i = 0; i < n; ++i) *reinterpret_cast<float4*>(x + i * ld_x + c) = v;
         const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int e = 0; e < E; ++e) {
+        for (int e = 0; e < rows; ++e) {
             *reinterpret_cast<float4*>(msg_a + e * ld_m + c) = zero;
             if (msg_b) *reinterpret_cast<float4*>(msg_b + e * ld_m + c) = zero;
         }
@@ -905,6 +983,21 @@ __global__ void relay_fill_mu_kernel(float* mu, const float* mix, int n, int K, 
             const float4 sv = scale4_rn(acc, scale);
             *reinterpret_cast<float4*>(mu + i * ld_x + c) =
                 make_float4(sv.x, c + 1 < d ? sv.y : 0.f, c + 2 < d ? sv.z : 0.f, c + 3 < d ? sv.w : 0.f);
+        }
+    }
+}
+
+// The K Gaussian centres N_k themselves ([K][ld_x], Philox stream 1, row k),
+// as relay_fill_mu_kernel draws them; ragged columns beyond d are zero.
+__global__ void relay_fill_centres_kernel(float* centres, int K, int64_t ld_x, int64_t nquads, int64_t d,
+                                          uint32_t q0, const __grid_constant__ PhiloxKey key) {
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < nquads; q += stride) {
+        const int64_t c = 4 * q;
+        for (int k = 0; k < K; ++k) {
+            const float4 z = normal4(q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k), 0u, 1u, key);
+            *reinterpret_cast<float4*>(centres + k * ld_x + c) =
+                make_float4(z.x, c + 1 < d ? z.y : 0.f, c + 2 < d ? z.z : 0.f, c + 3 < d ? z.w : 0.f);
         }
     }
 }
@@ -1096,23 +1189,50 @@ int resident_ctas(int dev, int threads, size_t smem) {
     return per_sm;
 }
 
-template <int OBJ, int OPT>
-int launch_models(const relay_handle* h, const ModelArgs& a, cudaStream_t stream, bool after_counts) {
+// The walk over NT handles' windows in one launch (NT = 1: one handle).  The
+// handles share the objective source and the local optimiser (the caller
+// checks); threads and shared memory are sized for the larger program, and
+// the CTAs are split between the windows in proportion to their quads.
+template <int OBJ, int OPT, int NT, bool WIDE>
+int launch_models(const relay_handle* const* hs, const ModelArgs* as, cudaStream_t stream, bool after_counts) {
     int dev = 0;
     const int sms = device_sms(&dev);
     if (sms <= 0) return RELAY_ECUDA;
-    const int per_thread = h->prog.nslots + (OBJ == relaysum::kMuCachedCentres ? h->obj.K : 0);
+    int per_thread = 0;
+    for (int k = 0; k < NT; ++k)
+        per_thread = std::max(per_thread, hs[k]->prog.nslots + (OBJ == relaysum::kMuCachedCentres ||
+                                                                OBJ == relaysum::kMuStoredCentres ? hs[k]->obj.K : 0));
     const int threads = models_threads(per_thread);
     const size_t smem = static_cast<size_t>(per_thread) * threads * 16;
     if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
-    const int per_sm = resident_ctas<relay_models_kernel<OBJ, OPT>>(dev, threads, smem);
+    const int per_sm = resident_ctas<relay_models_kernel<OBJ, OPT, NT, WIDE>>(dev, threads, smem);
     if (per_sm <= 0) return RELAY_ECUDA;
-    const int64_t want = (a.nquads + threads - 1) / threads;
     const int64_t cap = static_cast<int64_t>(sms) * per_sm;
-    const int grid = static_cast<int>(want < cap ? want : cap);
-    const PhiloxKey mu_key = philox_key(static_cast<uint64_t>(h->obj.k0) | (static_cast<uint64_t>(h->obj.k1) << 32));
-    return launch_step_kernel(relay_models_kernel<OBJ, OPT>, grid, threads, smem, stream, after_counts, h->prog,
-                              h->obj, mu_key, a);
+    int64_t want[NT], total = 0, nq = 0;
+    for (int k = 0; k < NT; ++k) {
+        want[k] = (as[k].nquads + threads - 1) / threads;
+        total += want[k];
+        nq += as[k].nquads;
+    }
+    Windows<NT> win;
+    for (int k = 0; k < NT; ++k) {
+        win.prog[k] = hs[k]->prog;
+        win.a[k] = as[k];
+    }
+    int64_t grid = total < cap ? total : cap;
+    win.split = 0;
+    if (NT == 2) {
+        int64_t split = want[0];
+        if (total > cap) {  // CTAs in proportion to the quads, at least one per window
+            split = (cap * as[0].nquads + nq / 2) / nq;
+            split = std::min(std::max<int64_t>(split, 1), cap - 1);
+        }
+        win.split = static_cast<int32_t>(split);
+    }
+    const PhiloxKey mu_key =
+        philox_key(static_cast<uint64_t>(hs[0]->obj.k0) | (static_cast<uint64_t>(hs[0]->obj.k1) << 32));
+    return launch_step_kernel(relay_models_kernel<OBJ, OPT, NT, WIDE>, static_cast<int>(grid), threads, smem, stream,
+                              after_counts, win, hs[0]->obj, mu_key);
 }
 
 // Quads per CTA of the node-parallel kernel, threads = qb * n <= 1024: a
@@ -1153,18 +1273,42 @@ bool use_nodes(const relay_handle* h) {
     return true;
 }
 
+// Whether a tree has a node of degree > kRegDeg (the walk's WIDE variant).
+bool has_wide(const relay_handle* h) {
+    for (int i = 0; i < h->prog.n; ++i)
+        if (h->prog.node[i].deg > kRegDeg) return true;
+    return false;
+}
+
+template <int OPT, int NT, bool WIDE>
+int launch_walk_src(const relay_handle* const* hs, const ModelArgs* as, cudaStream_t stream, bool after_counts) {
+    switch (hs[0]->obj.source) {
+        case relaysum::kMuStored: return launch_models<relaysum::kMuStored, OPT, NT, WIDE>(hs, as, stream, after_counts);
+        case relaysum::kMuPerRow: return launch_models<relaysum::kMuPerRow, OPT, NT, WIDE>(hs, as, stream, after_counts);
+        case relaysum::kMuStoredCentres:
+            return launch_models<relaysum::kMuStoredCentres, OPT, NT, WIDE>(hs, as, stream, after_counts);
+        default: return launch_models<relaysum::kMuCachedCentres, OPT, NT, WIDE>(hs, as, stream, after_counts);
+    }
+}
+
+// One handle: the WIDE variant when its tree has a wide node.  Several
+// windows (relay_step_windows) launch together only when none has one.
+template <int OPT, int NT>
+int launch_walk_obj(const relay_handle* const* hs, const ModelArgs* as, cudaStream_t stream, bool after_counts) {
+    if (NT == 1 && has_wide(hs[0])) return launch_walk_src<OPT, 1, true>(hs, as, stream, after_counts);
+    return launch_walk_src<OPT, NT, false>(hs, as, stream, after_counts);
+}
+
 template <int OPT>
 int launch_models_obj(const relay_handle* h, const ModelArgs& a, cudaStream_t stream, bool after_counts) {
     if (use_nodes(h)) {
         if (h->obj.source == relaysum::kMuStored)
             return launch_nodes<relaysum::kMuStored, OPT>(h, a, stream, after_counts);
+        if (h->obj.source == relaysum::kMuStoredCentres)
+            return launch_nodes<relaysum::kMuStoredCentres, OPT>(h, a, stream, after_counts);
         return launch_nodes<relaysum::kMuPerRow, OPT>(h, a, stream, after_counts);
     }
-    switch (h->obj.source) {
-        case relaysum::kMuStored: return launch_models<relaysum::kMuStored, OPT>(h, a, stream, after_counts);
-        case relaysum::kMuPerRow: return launch_models<relaysum::kMuPerRow, OPT>(h, a, stream, after_counts);
-        default: return launch_models<relaysum::kMuCachedCentres, OPT>(h, a, stream, after_counts);
-    }
+    return launch_walk_obj<OPT, 1>(&h, &a, stream, after_counts);
 }
 
 // Quads per CTA of relay_fused_steps_kernel: nodes_qb, halved (down to 4)
@@ -1203,6 +1347,7 @@ int launch_fused(const relay_handle* h, const ModelArgs& a, const FusedSteps& fs
 // and d = 4096 to 32 workers and d = 1.1e8, the multi-step kernel was ahead
 // everywhere (1.2x to 1.8x).
 bool use_fused(const relay_handle* h) {
+    if (h->prog.nwide > 0) return false;  // received-sum rows are kept by the per-step kernels only
     if (h->kernel == RELAY_KERNEL_NODES) return true;
     if (h->kernel == RELAY_KERNEL_WALK) return false;
     for (int i = 0; i < h->prog.n; ++i)
@@ -1213,8 +1358,14 @@ bool use_fused(const relay_handle* h) {
 template <int OPT>
 int launch_fused_obj(const relay_handle* h, const ModelArgs& a, const FusedSteps& fs, cudaStream_t stream) {
     if (h->obj.source == relaysum::kMuStored) return launch_fused<relaysum::kMuStored, OPT>(h, a, fs, stream);
+    if (h->obj.source == relaysum::kMuStoredCentres)
+        return launch_fused<relaysum::kMuStoredCentres, OPT>(h, a, fs, stream);
     return launch_fused<relaysum::kMuPerRow, OPT>(h, a, fs, stream);
 }
+
+// Rows of a message buffer: E, plus one received-sum row per wide node when
+// received sums are on.
+int message_rows(const relay_handle* h) { return h->prog.E + h->prog.nwide; }
 
 // Argument checks shared by relay_step_models and relay_step.
 int check_step_args(const relay_handle* h, const float* x, const float* msg_in, const float* msg_out,
@@ -1222,6 +1373,7 @@ int check_step_args(const relay_handle* h, const float* x, const float* msg_in, 
     if (!h || !h->has_objective || !std::isfinite(lr)) return RELAY_EINVAL;
     if (step < 0 || step >= (int64_t(1) << 32)) return RELAY_EINVAL;
     const int E = h->prog.E;
+    const int rows = message_rows(h);
     if (E > 0 && !counts) return RELAY_EINVAL;
     if (h->d == 0) return RELAY_OK;  // counters only
     if (E > 0 && (!msg_in || !msg_out || msg_in == msg_out)) return RELAY_EINVAL;
@@ -1229,7 +1381,7 @@ int check_step_args(const relay_handle* h, const float* x, const float* msg_in, 
         return RELAY_EINVAL;
     // exact byte spans of the strided arrays (windows of wider arrays may sit side by side)
     const int64_t xb = ((h->prog.n - 1) * h->ld_x + 4 * h->nquads) * 4;
-    const int64_t mb = E > 0 ? ((E - 1) * h->ld_m + 4 * h->nquads) * 4 : 0;
+    const int64_t mb = rows > 0 ? ((rows - 1) * h->ld_m + 4 * h->nquads) * 4 : 0;
     if (overlap(x, xb, msg_in, mb) || overlap(x, xb, msg_out, mb) || overlap(msg_in, mb, msg_out, mb))
         return RELAY_EINVAL;
     for (const float* st : {static_cast<const float*>(h->s1), static_cast<const float*>(h->s2)})
@@ -1244,6 +1396,16 @@ int grid_for(int64_t items, int threads) {
     const int64_t want = (items + threads - 1) / threads;
     const int64_t cap = static_cast<int64_t>(sms > 0 ? sms : 1) * 8;
     return static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
+}
+
+// Window k of a counter launch: handle h's program, lost mask and arrays.
+template <int NT>
+void count_window(const relay_handle* h, int32_t* counts, CountWindows<NT>& cw, int k) {
+    cw.prog[k] = h->prog;
+    std::memcpy(cw.lost[k].w, h->lost, sizeof(cw.lost[k].w));
+    cw.has_lost[k] = h->has_lost ? 1 : 0;
+    cw.counts[k] = counts;
+    cw.dme_count[k] = h->algo == RELAY_ALGO_DME ? h->dme_count : nullptr;
 }
 
 }  // namespace
@@ -1354,6 +1516,35 @@ int relay_set_kernel(relay_handle* h, int32_t kernel) {
     return RELAY_OK;
 }
 
+int relay_set_received_sums(relay_handle* h, int32_t enable) {
+    if (!h || (enable != 0 && enable != 1)) return RELAY_EINVAL;
+    if ((enable != 0) == h->rsum) return RELAY_OK;
+    // rebuild the visit program from the handle's own edge list (edge 2u is
+    // the u-th pair as given)
+    const int n = h->prog.n;
+    int32_t edges[2 * (kMaxN - 1)];
+    for (int u = 0; u < n - 1; ++u) {
+        edges[2 * u] = h->prog.edge_src[2 * u];
+        edges[2 * u + 1] = h->prog.edge_dst[2 * u];
+    }
+    Program* p = new (std::nothrow) Program;
+    if (!p) return RELAY_ENOMEM;
+    int rc = RELAY_OK;
+    try {
+        rc = relaysum::build_program(n, edges, n - 1, p, enable != 0);
+    } catch (...) {
+        rc = RELAY_ENOMEM;
+    }
+    if (rc == RELAY_OK) {
+        h->prog = *p;
+        h->rsum = enable != 0;
+    }
+    delete p;
+    return rc;
+}
+
+int32_t relay_message_rows(const relay_handle* h) { return h ? message_rows(h) : RELAY_EINVAL; }
+
 int relay_get_kernel(const relay_handle* h) {
     if (!h) return RELAY_EINVAL;
     return use_nodes(h) ? RELAY_KERNEL_NODES : RELAY_KERNEL_WALK;
@@ -1376,31 +1567,40 @@ int relay_set_objective(relay_handle* h, const float* mu, float sigma) {
     return RELAY_OK;
 }
 
-int relay_set_objective_generated(relay_handle* h, const float* mix, int32_t K, float mu_scale,
-                                  uint64_t mu_seed, float sigma) {
-    if (!h || K < 0 || (K > 0 && !mix) || !std::isfinite(mu_scale) || !std::isfinite(sigma) ||
-        sigma < 0.0f)
-        return RELAY_EINVAL;
+// The non-zeros of a host mixture matrix mix [n][K] into an Objective.
+static int mixture(const relay_handle* h, const float* mix, int32_t K, float mu_scale, Objective* o, int* nnz_out) {
     if (K > 32767) return RELAY_EUNSUPPORTED;
     const int n = h->prog.n;
-    Objective o;
-    std::memset(&o, 0, sizeof(o));
+    std::memset(o, 0, sizeof(*o));
     int nnz = 0;
     for (int i = 0; i < n; ++i) {
-        o.row_off[i] = static_cast<int16_t>(nnz);
+        o->row_off[i] = static_cast<int16_t>(nnz);
         for (int k = 0; k < K; ++k) {
             const float w = mix[static_cast<int64_t>(i) * K + k];
             if (!std::isfinite(w)) return RELAY_EINVAL;
             if (w == 0.0f) continue;
             if (nnz >= relaysum::kMaxMixNnz) return RELAY_EUNSUPPORTED;
-            o.col[nnz] = static_cast<int16_t>(k);
-            o.w[nnz] = w;
+            o->col[nnz] = static_cast<int16_t>(k);
+            o->w[nnz] = w;
             ++nnz;
         }
     }
-    o.row_off[n] = static_cast<int16_t>(nnz);
-    o.K = K;
-    o.scale = mu_scale;
+    o->row_off[n] = static_cast<int16_t>(nnz);
+    o->K = K;
+    o->scale = mu_scale;
+    *nnz_out = nnz;
+    return RELAY_OK;
+}
+
+int relay_set_objective_generated(relay_handle* h, const float* mix, int32_t K, float mu_scale,
+                                  uint64_t mu_seed, float sigma) {
+    if (!h || K < 0 || (K > 0 && !mix) || !std::isfinite(mu_scale) || !std::isfinite(sigma) ||
+        sigma < 0.0f)
+        return RELAY_EINVAL;
+    Objective o;
+    int nnz = 0;
+    const int rc = mixture(h, mix, K, mu_scale, &o, &nnz);
+    if (rc != RELAY_OK) return rc;
     o.k0 = static_cast<uint32_t>(mu_seed);
     o.k1 = static_cast<uint32_t>(mu_seed >> 32);
     // one Philox block per non-zero, or K per quad when that is fewer
@@ -1408,6 +1608,24 @@ int relay_set_objective_generated(relay_handle* h, const float* mix, int32_t K, 
                                                               : relaysum::kMuPerRow;
     h->obj = o;
     h->mu = nullptr;
+    h->sigma = sigma;
+    h->has_objective = true;
+    return RELAY_OK;
+}
+
+int relay_set_objective_centres(relay_handle* h, const float* centres, const float* mix, int32_t K,
+                                float mu_scale, float sigma) {
+    if (!h || K < 1 || !mix || !std::isfinite(mu_scale) || !std::isfinite(sigma) || sigma < 0.0f)
+        return RELAY_EINVAL;
+    if (h->d > 0 && (!centres || !aligned16(centres))) return RELAY_EINVAL;
+    if (K > relaysum::kMaxCachedCentres) return RELAY_EUNSUPPORTED;
+    Objective o;
+    int nnz = 0;
+    const int rc = mixture(h, mix, K, mu_scale, &o, &nnz);
+    if (rc != RELAY_OK) return rc;
+    o.source = relaysum::kMuStoredCentres;
+    h->obj = o;
+    h->mu = centres;
     h->sigma = sigma;
     h->has_objective = true;
     return RELAY_OK;
@@ -1422,6 +1640,16 @@ int relay_fill_objective(relay_handle* h, float* mu, const float* mix, int32_t K
     relay_fill_mu_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
         mu, mix, h->prog.n, K, h->ld_x, h->nquads, h->d, static_cast<uint32_t>(h->c0 / 4), mu_scale,
         philox_key(mu_seed));
+    return launch_status();
+}
+
+int relay_fill_centres(relay_handle* h, float* centres, int32_t K, uint64_t mu_seed, relay_stream_t stream) {
+    if (!h || K < 1) return RELAY_EINVAL;
+    if (h->d == 0) return RELAY_OK;
+    if (!centres || !aligned16(centres)) return RELAY_EINVAL;
+    const int threads = 256;
+    relay_fill_centres_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
+        centres, K, h->ld_x, h->nquads, h->d, static_cast<uint32_t>(h->c0 / 4), philox_key(mu_seed));
     return launch_status();
 }
 
@@ -1445,7 +1673,7 @@ int relay_init(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* c
             return RELAY_ECUDA;
     const int threads = 256;
     relay_init_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
-        x, E > 0 ? msg_a : nullptr, E > 0 ? msg_b : nullptr, h->prog.n, E, h->ld_x, h->ld_m, h->nquads,
+        x, E > 0 ? msg_a : nullptr, E > 0 ? msg_b : nullptr, h->prog.n, message_rows(h), h->ld_x, h->ld_m, h->nquads,
         h->d, static_cast<uint32_t>(h->c0 / 4), x0_std, philox_key(seed));
     return launch_status();
 }
@@ -1454,10 +1682,9 @@ int relay_step_counts(relay_handle* h, int32_t* counts, relay_stream_t stream) {
     if (!h) return RELAY_EINVAL;
     if (h->prog.E == 0 && h->algo != RELAY_ALGO_DME) return RELAY_OK;
     if (!counts && h->prog.E > 0) return RELAY_EINVAL;
-    LostMask lost;
-    std::memcpy(lost.w, h->lost, sizeof(lost.w));
-    relay_counts_kernel<<<1, 256, 0, stream>>>(h->prog, lost, h->has_lost ? 1 : 0, counts,
-                                               h->algo == RELAY_ALGO_DME ? h->dme_count : nullptr);
+    CountWindows<1> cw;
+    count_window(h, counts, cw, 0);
+    relay_counts_kernel<1><<<1, 256, 0, stream>>>(cw);
     return launch_status();
 }
 
@@ -1491,6 +1718,7 @@ static ModelArgs model_args(const relay_handle* h, float* x, const float* msg_in
     a.mode = h->mode;
     a.algo = h->algo;
     a.has_lost = h->has_lost ? 1 : 0;
+    a.rsum = h->prog.nwide > 0 ? 1 : 0;
     std::memcpy(a.lost.w, h->lost, sizeof(a.lost.w));
     a.s1 = h->s1;
     a.s2 = h->s2;
@@ -1536,6 +1764,58 @@ int relay_step(relay_handle* h, float* x, const float* msg_in, float* msg_out, i
     return step_models(h, x, msg_in, msg_out, counts, lr, seed, step, stream, counted);
 }
 
+// relay_step_windows runs the windows in one launch when both take the walk,
+// neither tree has a node of degree > kRegDeg (double binary trees have
+// degree <= 3), and they share the objective (its source; the mixture too
+// when regenerated) and the local optimiser; otherwise it issues one
+// relay_step per window.
+static bool one_launch(const relay_handle* a, const relay_handle* b) {
+    if (a->d == 0 || b->d == 0 || use_nodes(a) || use_nodes(b) || has_wide(a) || has_wide(b)) return false;
+    if (a->opt != b->opt || a->obj.source != b->obj.source) return false;
+    return a->obj.source == relaysum::kMuStored || std::memcmp(&a->obj, &b->obj, sizeof(Objective)) == 0;
+}
+
+int relay_step_windows(relay_handle* const* h, int32_t count, float* const* x, const float* const* msg_in,
+                       float* const* msg_out, int32_t* const* counts, float lr, uint64_t seed, int64_t step,
+                       relay_stream_t stream) {
+    if (!h || !x || !msg_in || !msg_out || !counts || count < 1 || count > RELAY_MAX_WINDOWS) return RELAY_EINVAL;
+    for (int k = 0; k < count; ++k) {
+        if (!h[k]) return RELAY_EINVAL;
+        for (int j = 0; j < k; ++j)
+            if (h[j] == h[k]) return RELAY_EINVAL;
+        const int rc = check_step_args(h[k], x[k], msg_in[k], msg_out[k], counts[k], lr, step);
+        if (rc != RELAY_OK) return rc;
+    }
+    if (count == 1 || !one_launch(h[0], h[1])) {
+        for (int k = 0; k < count; ++k) {
+            const int rc = relay_step(h[k], x[k], msg_in[k], msg_out[k], counts[k], lr, seed, step, stream);
+            if (rc != RELAY_OK) return rc;
+        }
+        return RELAY_OK;
+    }
+    // the counters of both windows (one CTA each), then the step kernel as
+    // its programmatic dependent
+    bool counted = false;
+    CountWindows<2> cw;
+    for (int k = 0; k < 2; ++k) {
+        count_window(h[k], counts[k], cw, k);
+        counted = counted || h[k]->prog.E > 0 || h[k]->algo == RELAY_ALGO_DME;
+    }
+    if (counted) {
+        relay_counts_kernel<2><<<2, 256, 0, stream>>>(cw);
+        const int rc = launch_status();
+        if (rc != RELAY_OK) return rc;
+    }
+    const ModelArgs as[2] = {model_args(h[0], x[0], msg_in[0], msg_out[0], counts[0], lr, seed, step),
+                             model_args(h[1], x[1], msg_in[1], msg_out[1], counts[1], lr, seed, step)};
+    const relay_handle* const hs[2] = {h[0], h[1]};
+    switch (h[0]->opt) {
+        case 0: return launch_walk_obj<0, 2>(hs, as, stream, counted);
+        case 1: return launch_walk_obj<1, 2>(hs, as, stream, counted);
+        default: return launch_walk_obj<2, 2>(hs, as, stream, counted);
+    }
+}
+
 int relay_get_steps_kernel(const relay_handle* h) {
     if (!h) return RELAY_EINVAL;
     return use_fused(h) ? RELAY_KERNEL_FUSED : relay_get_kernel(h);
@@ -1577,7 +1857,7 @@ int relay_steps(relay_handle* h, float* x, float* msg_a, float* msg_b, int32_t* 
         }
         // the counters advance after the models kernel, which read them
         if (counted) {
-            relay_counts_steps_kernel<<<1, 256, 0, stream>>>(h->prog, lost, h->has_lost ? 1 : 0, counts,
+            relay_counts_steps_kernel<<<1, kCountsThreads, 0, stream>>>(h->prog, lost, h->has_lost ? 1 : 0, counts,
                                                              h->algo == RELAY_ALGO_DME ? h->dme_count : nullptr, kc);
             rc = launch_status();
             if (rc != RELAY_OK) return rc;
@@ -1607,9 +1887,10 @@ int relay_program(const relay_handle* h, int32_t* nslots, int32_t* order, int32_
         if (order) order[i] = p.order[i];
         if (node_rec) {
             const NodeRec& r = p.node[i];
-            const int32_t v[10] = {r.deg,        r.pos_base,   r.parent_pos, r.recv_slot, r.acc_slot,
-                                   r.parent_acc, r.fin_parent, r.parent,     r.tot_slot,  r.flags};
-            std::memcpy(node_rec + 10 * i, v, sizeof(v));
+            const int32_t v[12] = {r.deg,        r.pos_base,   r.parent_pos, r.recv_slot, r.acc_slot,
+                                   r.parent_acc, r.fin_parent, r.parent,     r.tot_slot,  r.flags,
+                                   p.rsum_slot[i], p.rsum_row[i]};
+            std::memcpy(node_rec + 12 * i, v, sizeof(v));
         }
     }
     if (pos_rec)
@@ -1644,6 +1925,10 @@ int relay_metrics(relay_handle* h, const float* x, double* workspace, double* ou
     switch (h->obj.source) {
         case relaysum::kMuStored:
             relay_metrics_kernel<relaysum::kMuStored><<<blocks, kMetricsThreads, 0, stream>>>(
+                h->obj, mu_key, a, n, h->d, workspace);
+            break;
+        case relaysum::kMuStoredCentres:
+            relay_metrics_kernel<relaysum::kMuStoredCentres><<<blocks, kMetricsThreads, 0, stream>>>(
                 h->obj, mu_key, a, n, h->d, workspace);
             break;
         default:  // cached centres are regenerated per row here

@@ -18,20 +18,26 @@ from . import _native as nat
 
 def lr_correction(n: int, edges, mode: int = 1, tol: float = 1e-7, max_steps: int = 100_000,
                   device="cuda"):
-    """Returns (alpha_n, the per-worker limits [n]) for the given tree."""
+    """Returns (alpha_n, the per-worker limits [n]) for the given tree.
+    Raises RuntimeError if the models still move by more than `tol` after
+    `max_steps` steps (the limit was not reached)."""
     import torch
     run = nat.RelayRun(n, 4, edges, device=device, mode=mode)
     run.init(0.0, 0, np.zeros((n, 1), np.float32), 0.0, 0, 0.0)   # x^0 = 0
     run.mu.fill_(1.0)                                             # one update of +1:
     run.step(1.0, 0)                                              # x - 1 (x - mu) = 1
     prev = run.x[:, 0].clone()
+    converged = False
     for k in range(max_steps):
         run.step(0.0, 0)                                          # no further updates
         if k % 64 == 63:
             cur = run.x[:, 0].clone()
             if float((cur - prev).abs().max()) <= tol:
+                converged = True
                 break
             prev = cur
+    if not converged:
+        raise RuntimeError(f"lr_correction: models still moving by more than {tol} after {max_steps} steps")
     torch.cuda.synchronize(run.device)
     limits = run.x[:, 0].double().cpu().numpy()
     return float(limits.mean()), limits

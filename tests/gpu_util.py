@@ -4,6 +4,9 @@ chosen coordinates, compare with the parity metric.
 Parity metric (per array, padding excluded):
     max_e |g_e - r_e| / max(|r_e|, rms(r))  <=  1e-5
 with g the fp32 GPU value and r the fp64 oracle value; counters must be equal.
+parity_report adds the plain errors beside it (max absolute, max relative,
+and how many elements sit below the rms floor); the full-size tests record
+them when RELAY_PARITY_LOG names a file.
 The fp32 path differs from the fp64 definition only by rounding: a float32
 restatement of the step stays within 1e-6 of the oracle on every workload
 (10x below the bar), so 1e-5 leaves room for the GPU's own summation order
@@ -21,6 +24,10 @@ from oracle import oracle
 
 RTOL = 1e-5
 
+# When set, the full-size parity tests append one JSON line per compared
+# array to this file: the metric above and the plain errors beside it.
+PARITY_LOG = os.environ.get("RELAY_PARITY_LOG")
+
 
 def parity_error(g: np.ndarray, r: np.ndarray) -> float:
     g = np.asarray(g, dtype=np.float64)
@@ -30,6 +37,50 @@ def parity_error(g: np.ndarray, r: np.ndarray) -> float:
     rms = float(np.sqrt(np.mean(r * r)))
     denom = np.maximum(np.abs(r), rms if rms > 0 else 1.0)
     return float(np.max(np.abs(g - r) / denom))
+
+
+def parity_report(g: np.ndarray, r: np.ndarray) -> dict:
+    """The parity metric with the plain errors beside it:
+    floored        max |g - r| / max(|r|, rms(r)) (the bar, 1e-5);
+    abs_max        max |g - r|;
+    rel_max        max |g - r| / |r| over the elements with r != 0;
+    rel_max_at     |r| / rms(r) at that element (how close to zero it sits);
+    rel_max_big    max |g - r| / |r| over the elements with |r| >= rms(r),
+                   where the two metrics coincide;
+    floor_share    the fraction of elements whose denominator is the rms
+                   floor (|r| < rms(r)) rather than |r|;
+    over_bar_share the fraction whose plain relative error exceeds 1e-5."""
+    g = np.asarray(g, dtype=np.float64).ravel()
+    r = np.asarray(r, dtype=np.float64).ravel()
+    out = {"elements": int(r.size)}
+    if r.size == 0:
+        return out
+    diff = np.abs(g - r)
+    rms = float(np.sqrt(np.mean(r * r)))
+    a = np.abs(r)
+    out["rms"] = rms
+    out["floored"] = float(np.max(diff / np.maximum(a, rms if rms > 0 else 1.0)))
+    out["abs_max"] = float(diff.max())
+    nz = a > 0
+    if nz.any():
+        rel = diff[nz] / a[nz]
+        k = int(np.argmax(rel))
+        out["rel_max"] = float(rel[k])
+        out["rel_max_at"] = float(a[nz][k] / rms) if rms > 0 else None
+        out["over_bar_share"] = float(np.mean(rel > RTOL)) * float(nz.mean())
+    big = a >= rms
+    out["rel_max_big"] = float(np.max(diff[big] / a[big])) if big.any() else None
+    out["floor_share"] = float(np.mean(a < rms))
+    return out
+
+
+def record_parity(label: str, array: str, g, r):
+    """Appends parity_report(g, r) for `array` of case `label` to PARITY_LOG (if set)."""
+    if not PARITY_LOG:
+        return
+    import json
+    with open(PARITY_LOG, "a") as f:
+        f.write(json.dumps({"case": label, "array": array, **parity_report(g, r)}) + "\n")
 
 
 def gpu_run(w, steps: int, mode: int | None = None, d: int | None = None, c0: int = 0,
@@ -100,9 +151,11 @@ def oracle_ranges(w, ranges, steps: int, mode: int | None = None, c0: int = 0) -
     return parallel_map(lambda r: oracle_range(w, c0 + r[0], r[1], steps, mode), ranges)
 
 
-def compare_ranges(run: rs.RelayRun, w, ranges, steps: int, mode: int | None = None, c0: int = 0):
+def compare_ranges(run: rs.RelayRun, w, ranges, steps: int, mode: int | None = None, c0: int = 0,
+                   label: str | None = None):
     """Max parity error of x and of the last messages over the given ranges;
-    asserts the counters are bit-exact."""
+    asserts the counters are bit-exact.  With a label, the plain errors are
+    recorded too (record_parity)."""
     gx, gm, ox, om = [], [], [], []
     counts = None
     for (start, length), st in zip(ranges, oracle_ranges(w, ranges, steps, mode, c0)):
@@ -113,8 +166,16 @@ def compare_ranges(run: rs.RelayRun, w, ranges, steps: int, mode: int | None = N
         counts = st.counts
     g_counts = run.counts[:run.E].cpu().numpy()
     assert np.array_equal(g_counts, counts), (g_counts, counts)
-    ex = parity_error(np.concatenate(gx, axis=1), np.concatenate(ox, axis=1))
-    em = parity_error(np.concatenate(gm, axis=1), np.concatenate(om, axis=1)) if run.E else 0.0
+    gx, ox = np.concatenate(gx, axis=1), np.concatenate(ox, axis=1)
+    ex = parity_error(gx, ox)
+    em = 0.0
+    if run.E:
+        gm, om = np.concatenate(gm, axis=1), np.concatenate(om, axis=1)
+        em = parity_error(gm, om)
+    if label:
+        record_parity(label, "x", gx, ox)
+        if run.E:
+            record_parity(label, "messages", gm, om)
     return ex, em
 
 

@@ -2,7 +2,8 @@
 init, steps, allocation-free metrics, destroy), compiled against the
 library, must give the same models bit for bit as the Python binding's run of
 the same configuration, and the same metrics -- with the C program stepping
-through relay_step calls or through one relay_steps call."""
+through relay_step calls, through one relay_steps call, or through
+relay_step_host calls on a state in page-locked host memory."""
 import os
 import subprocess
 
@@ -31,13 +32,13 @@ def c_program(tmp_path_factory):
     return exe, os.path.dirname(lib)
 
 
-@pytest.mark.parametrize("fused", [False, True])
+@pytest.mark.parametrize("path", ["step", "fused", "host"])
 @pytest.mark.parametrize("tree,n,d,steps,mode", [("chain", 8, 4096, 100, 1), ("binary", 16, 70001, 30, 0)])
-def test_c_program_equals_python_binding(c_program, tmp_path, tree, n, d, steps, mode, fused):
+def test_c_program_equals_python_binding(c_program, tmp_path, tree, n, d, steps, mode, path):
     exe, libdir = c_program
     out = tmp_path / "out.bin"
     env = dict(os.environ, LD_LIBRARY_PATH=libdir + os.pathsep + os.environ.get("LD_LIBRARY_PATH", ""))
-    r = subprocess.run([exe, tree, str(n), str(d), str(steps), str(mode), str(out)] + (["fused"] if fused else []),
+    r = subprocess.run([exe, tree, str(n), str(d), str(steps), str(mode), str(out)] + ([] if path == "step" else [path]),
                        env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0, r.stderr
     raw = out.read_bytes()

@@ -11,7 +11,7 @@ import paper_2110_04175_gb300 as rs
 from oracle import oracle
 from paper_2110_04175_gb300 import build as rs_build
 from paper_2110_04175_gb300 import workloads as wl
-from tests.gpu_util import RTOL, adam_step_bound, c8_sample, parallel_map, parity_error
+from tests.gpu_util import RTOL, adam_step_bound, c8_sample, parallel_map, parity_error, record_parity
 
 pytestmark = pytest.mark.gpu
 
@@ -29,7 +29,7 @@ def _gpu():
     torch.cuda.empty_cache()
 
 
-def _run_both(w, steps, mode, optimizer=None, lost=None, ranges=None, objective="stored"):
+def _run_both(w, steps, mode, optimizer=None, lost=None, ranges=None, objective="stored", label=None):
     """GPU run through the C ABI and oracle runs on `ranges` (default: all
     coordinates); lost: [steps][E] flags or None.  Returns the parity errors."""
     run = rs.RelayRun(w.n, w.d, w.edges, device="cuda:0", mode=mode, objective=objective,
@@ -72,6 +72,9 @@ def _run_both(w, steps, mode, optimizer=None, lost=None, ranges=None, objective=
     del run
     gc.collect()
     torch.cuda.empty_cache()
+    if label:
+        record_parity(label, "x", gx, ox)
+        record_parity(label, "messages", gm, om)
     return parity_error(gx, ox), parity_error(gm, om)
 
 
@@ -93,7 +96,7 @@ def test_nesterov_full_size_sampled():
     steps), oracle on the first and last 65,536 coordinates and 1,024 random
     windows of 1,024."""
     w = wl.binary32_bert()
-    ex, em = _run_both(w, w.steps, w.mode, "nesterov", ranges=c8_sample(w.d, seed=5))
+    ex, em = _run_both(w, w.steps, w.mode, "nesterov", ranges=c8_sample(w.d, seed=5), label=f"{w.name}/nesterov")
     assert ex <= RTOL and em <= RTOL, (ex, em)
 
 
@@ -139,6 +142,8 @@ def test_adam_full_size_sampled():
     ox = np.concatenate([r[0].x for r in res], 1)
     om = np.concatenate([r[0].msg for r in res], 1)
     bound = np.concatenate([r[1] for r in res])
+    record_parity(f"{w.name}/adam", "x", gx, ox)
+    record_parity(f"{w.name}/adam", "messages", gm, om)
     for g, r, scale in ((gx, ox, 1.0), (gm, om, float(w.n))):
         rms = float(np.sqrt(np.mean(r * r)))
         plain = RTOL * np.maximum(np.abs(r), rms)
@@ -170,7 +175,7 @@ def test_lost_messages_with_momentum_full_size_sampled():
                     1.0, 0.05, 0.05, 0.0, 60)
     lost = (np.random.default_rng(7).random((w.steps, w.E)) < 0.10).astype(np.uint8)
     ranges = c8_sample(w.d, seed=6)
-    ex, em = _run_both(w, w.steps, 1, "nesterov", lost=lost, ranges=ranges)
+    ex, em = _run_both(w, w.steps, 1, "nesterov", lost=lost, ranges=ranges, label=f"{w.name}/nesterov/lost")
     assert ex <= RTOL and em <= RTOL, (ex, em)
 
 
@@ -252,6 +257,8 @@ def test_other_algorithms_full_size_sampled(algorithm):
         gm.append(run.messages[:run.E, start:start + length].double().cpu().numpy())
         ox.append(st.x)
         om.append(st.msg)
+    record_parity(f"{w.name}/{algorithm}", "x", np.concatenate(gx, 1), np.concatenate(ox, 1))
+    record_parity(f"{w.name}/{algorithm}", "messages", np.concatenate(gm, 1), np.concatenate(om, 1))
     assert parity_error(np.concatenate(gx, 1), np.concatenate(ox, 1)) <= RTOL
     assert parity_error(np.concatenate(gm, 1), np.concatenate(om, 1)) <= RTOL
     del run

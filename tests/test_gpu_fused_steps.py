@@ -43,6 +43,10 @@ CASES = {
     "chain8_d4096": dict(n=8, edges=wl.chain(8), d=4096),
     "binary16_ragged_offset_alg1": dict(n=16, edges=wl.binary_tree(16), d=4097, c0=4000, mode=0),
     "star20_lost": dict(n=20, edges=wl.star(20), d=3001, lost_p=0.2),
+    # received sums off: under "nodes" the multi-step kernel's wide-node path
+    "star20_lost_plain": dict(n=20, edges=wl.star(20), d=3001, lost_p=0.2, received_sums=False),
+    "star64_dme_lost_plain": dict(n=64, edges=wl.star(64), d=513, algorithm="dme", lost_p=0.1,
+                                  received_sums=False),
     "random100_nesterov_generated": dict(n=100, edges=wl.random_tree(100, 7), d=333,
                                          optimizer=("nesterov", 0.9), objective="generated"),
     "binary200_adam": dict(n=200, edges=wl.binary_tree(200), d=65, optimizer=("adam", 0.9, 0.999, 1e-8)),
@@ -59,7 +63,8 @@ CASES = {
 def make_run(c, seed=3, kernel="auto"):
     run = rs.RelayRun(c["n"], c["d"], c["edges"], device="cuda:0", mode=c.get("mode", 1), c0=c.get("c0", 0),
                       objective=c.get("objective", "stored"), optimizer=c.get("optimizer"),
-                      algorithm=c.get("algorithm", "relaysgd"), kernel=kernel)
+                      algorithm=c.get("algorithm", "relaysgd"), kernel=kernel,
+                      received_sums=c.get("received_sums", True))
     n = c["n"]
     mix = wl.dirichlet_mix(n, 5, 0.3, seed) if n > 2 else wl.identity_mix(n)
     run.init(0.5, seed, mix, 1.5, seed + 1, 0.2)
@@ -79,8 +84,9 @@ def state_of(run):
     for t, tr in enumerate(run.trees):
         out[f"t{t}.cur"] = tr.cur
         if tr.E:
+            rows = rs.relay_message_rows(tr.h)  # the messages and any received-sum rows
             for b in (0, 1):
-                out[f"t{t}.msg{b}"] = tr.msg[b][:tr.E, :tr.d].clone()
+                out[f"t{t}.msg{b}"] = tr.msg[b][:rows, :tr.d].clone()
             out[f"t{t}.counts"] = tr.counts[:tr.E].clone()
         if tr.dme_count is not None:
             out[f"t{t}.dme"] = tr.dme_count.clone()
@@ -91,8 +97,9 @@ def state_of(run):
 @pytest.mark.parametrize("name", sorted(CASES))
 def test_steps_equal_step_calls_bit_for_bit(name, kernel):
     """kernel="nodes" forces the multi-step kernel for relay_steps (the wide-node
-    path included) and the node kernel for relay_step; under "auto" the stars
-    take the per-step fallback and the walk."""
+    path included, with received sums off) and the node kernel for relay_step;
+    under "auto", and with received sums on, the stars take the per-step
+    fallback."""
     c = CASES[name]
     a, b = make_run(c, kernel=kernel), make_run(c, kernel=kernel)
     lr, seed = 0.05, 11

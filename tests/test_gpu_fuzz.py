@@ -3,7 +3,8 @@
 Each case draws a tree (random, star, chain or binary; up to 100 workers), a
 vector length with a ragged tail, a coordinate offset, the rebuild rule, the
 centre source and mixture, the local optimiser, the algorithm, a rate of lost
-messages and the step kernel, then compares every coordinate of the models
+messages, the step kernel and whether the message buffers carry the wide
+nodes' received sums, then compares every coordinate of the models
 and messages, the counters (bit-exact) and the mean-estimation counts with
 the oracle.  Adam cases hold every element to the 1e-5 bar plus the fp32
 rounding bound derived from Adam's arithmetic (gpu_util.adam_step_bound,
@@ -60,7 +61,9 @@ def draw(case: int) -> dict:
                 kernel=str(rng.choice(["auto", "walk", "nodes"])), steps=int(rng.integers(3, 30)),
                 lr=float(rng.uniform(0.01, 0.3)), sigma=float(rng.uniform(0.0, 0.3)),
                 x0_std=float(rng.choice([0.0, 0.5])), mu_scale=float(rng.uniform(0.5, 3.0)),
-                seed=int(rng.integers(0, 2**40)), mu_seed=int(rng.integers(0, 2**40)))
+                seed=int(rng.integers(0, 2**40)), mu_seed=int(rng.integers(0, 2**40)),
+                # drawn from a stream of its own, so the other draws of each case are unchanged
+                received_sums=bool(np.random.default_rng(5000 + case).integers(0, 2)))
 
 
 @pytest.mark.parametrize("case", range(120))
@@ -70,7 +73,8 @@ def test_random_configuration_against_oracle(case):
     optimizer = {"sgd": None, "nesterov": ("nesterov", c["beta1"]),
                  "adam": ("adam", c["beta1"], c["beta2"], 1e-2)}[c["opt"]]
     run = rs.RelayRun(n, d, c["edges"], device="cuda:0", mode=c["mode"], c0=c["c0"],
-                      objective=c["objective"], optimizer=optimizer, algorithm=c["algo"], kernel=c["kernel"])
+                      objective=c["objective"], optimizer=optimizer, algorithm=c["algo"], kernel=c["kernel"],
+                      received_sums=c["received_sums"])
     run.init(c["x0_std"], c["seed"], c["mix"], c["mu_scale"], c["mu_seed"], c["sigma"])
     st = oracle.State(n, c["edges"], d, c0=c["c0"])
     st.init(c["x0_std"], c["seed"], c["mix"].astype(np.float64), c["mu_scale"], c["mu_seed"])

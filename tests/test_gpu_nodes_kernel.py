@@ -49,9 +49,10 @@ OPTIMIZERS = {None: None, "nesterov": ("nesterov", 0.9), "adam": ("adam", 0.9, 0
 
 
 def _run(kernel, n, edges, d, steps=12, mode=1, objective="stored", optimizer=None,
-         algorithm="relaysgd", lost_p=0.0, mix=None, seed=4):
+         algorithm="relaysgd", lost_p=0.0, mix=None, seed=4, received_sums=True):
     run = rs.RelayRun(n, d, edges, device="cuda:0", mode=mode, objective=objective,
-                      optimizer=OPTIMIZERS[optimizer], algorithm=algorithm, kernel=kernel)
+                      optimizer=OPTIMIZERS[optimizer], algorithm=algorithm, kernel=kernel,
+                      received_sums=received_sums)
     mix = wl.identity_mix(n) if mix is None else mix
     run.init(0.1, seed, mix, 1.0, seed + 1, 0.1)
     if algorithm == "dme":
@@ -71,7 +72,8 @@ def _assert_identical(a, b, d):
     for sa, sb in zip(a.state, b.state):
         assert torch.equal(sa[:, :d], sb[:, :d])
     for ta, tb in zip(a.trees, b.trees):
-        assert torch.equal(ta.messages[:ta.E, :ta.d], tb.messages[:tb.E, :tb.d])
+        rows = rs.relay_message_rows(ta.h)  # the messages and any received-sum rows
+        assert torch.equal(ta.messages[:rows, :ta.d], tb.messages[:rows, :tb.d])
         assert torch.equal(ta.counts[:ta.E], tb.counts[:tb.E])
         if ta.dme_count is not None:
             assert torch.equal(ta.dme_count, tb.dme_count)
@@ -103,6 +105,18 @@ def test_nodes_equal_walk_every_feature(shape, optimizer, algorithm, lost_p):
     n, edges = SHAPES[shape]
     _both(n, edges(), 2053, mode=0 if lost_p == 0 else 1, optimizer=optimizer,
           algorithm=algorithm, lost_p=lost_p)
+
+
+@pytest.mark.parametrize("objective", ["stored", "generated"])
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("shape", ["star9", "star64"])
+def test_nodes_equal_walk_wide_nodes_without_received_sums(shape, mode, objective):
+    """The wide path that reads every incoming row (received sums off)."""
+    n, edges = SHAPES[shape]
+    for d in (13, 4099):
+        _both(n, edges(), d, mode=mode, objective=objective, received_sums=False)
+    _both(n, edges(), 2053, optimizer="adam", lost_p=0.2, received_sums=False)
+    _both(n, edges(), 2053, algorithm="dme", lost_p=0.2, received_sums=False)
 
 
 @pytest.mark.parametrize("mix", ["dirichlet", "dense"])

@@ -20,7 +20,7 @@ from paper_2110_04175_gb300 import build as rs_build
 from paper_2110_04175_gb300 import workloads as wl
 from tests import treeutil as tu
 from tests.gpu_util import (RTOL, c8_sample, compare_ranges, gpu_run, oracle_range, parallel_map,
-                             parity_error, windows)
+                             parity_error, record_parity, windows)
 
 pytestmark = pytest.mark.gpu
 
@@ -116,7 +116,7 @@ def test_chain8_d4096_full_100_steps(mode, kernel):
     """The small workload, every coordinate, 100 steps, on each step kernel."""
     w = wl.chain8_d4096()
     run = gpu_run(w, w.steps, mode, kernel=kernel)
-    ex, em = compare_ranges(run, w, [(0, w.d)], w.steps, mode)
+    ex, em = compare_ranges(run, w, [(0, w.d)], w.steps, mode, label=f"{w.name}/{kernel}/mode{mode}")
     assert ex <= RTOL and em <= RTOL, (ex, em)
 
 
@@ -268,7 +268,7 @@ def test_full_size_workload_sampled(w):
     _free()
     run = gpu_run(w, w.steps, objective="stored")
     ranges = windows(w.d) if w.d < 1_000_000 else c8_sample(w.d, seed=w.n)
-    ex, em = compare_ranges(run, w, ranges, w.steps)
+    ex, em = compare_ranges(run, w, ranges, w.steps, label=w.name)
     del run
     _free()
     assert ex <= RTOL and em <= RTOL, (ex, em)
@@ -276,7 +276,8 @@ def test_full_size_workload_sampled(w):
 
 def test_double16_full_size_sampled():
     """Double binary trees (Section 3) at the VGG-11 size, 200 steps, as
-    bench.py runs them (stored centres, the two windows on forked streams).
+    bench.py runs them (stored centres, both windows in one relay_step_windows
+    launch).
     In each tree's coordinate window the oracle runs that tree on the first
     and last 65,536 coordinates and 1,024 random windows of 1,024."""
     _free()
@@ -299,6 +300,8 @@ def test_double16_full_size_sampled():
         ox = np.concatenate([st.x for st in states], 1)
         om = np.concatenate([st.msg for st in states], 1)
         assert np.array_equal(tr.counts[:tr.E].cpu().numpy(), states[0].counts)
+        record_parity(f"{w.name}/tree{run.trees.index(tr)}", "x", gx, ox)
+        record_parity(f"{w.name}/tree{run.trees.index(tr)}", "messages", gm, om)
         assert parity_error(gx, ox) <= RTOL and parity_error(gm, om) <= RTOL
     del run
     _free()
@@ -318,10 +321,10 @@ def test_binary16_resnet20_every_coordinate_mode0():
     assert np.array_equal(run.counts.cpu().numpy(), st.counts)
 
 
-def test_double_tree_steps_fork_and_join_in_graphs_and_eagerly():
-    """Double binary trees: RelayRun.step runs the two tree windows on forked
-    streams; the eager run, a CUDA graph of the same steps replayed once,
-    and steps issued window by window on one stream agree bit for bit."""
+def test_double_tree_steps_in_graphs_and_eagerly():
+    """Double binary trees: RelayRun.step runs both tree windows in one
+    relay_step_windows call; the eager run, a CUDA graph of the same steps
+    replayed once, and relay_step issued window by window agree bit for bit."""
     n, d = 16, 40_001
     trees = list(wl.double_binary_trees(n))
     runs = []

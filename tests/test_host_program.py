@@ -30,10 +30,15 @@ REG_DEG = 4
 
 def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0=0, lost=None):
     """One step executed the way relay_counts_kernel + relay_models_kernel do
-    (lost: E flags of messages lost in transit, or None)."""
+    (lost: E flags of messages lost in transit, or None).  With received sums
+    on (a wide node's rsum_row >= 0), msg_in and the result carry the sum
+    rows after the E message rows."""
     lost = np.zeros(2 * (n - 1), dtype=bool) if lost is None else np.asarray(lost, dtype=bool)
     nslots, order, node, pos = rs.relay_program(h)
     E = 2 * (n - 1)
+    sums = bool(n > 0 and (node[:, 11] >= 0).any())
+    rows = rs.relay_message_rows(h)
+    assert rows == E + int((node[:, 11] >= 0).sum())
     src, dst = rs.relay_edges(h)
     # counters
     counts = np.zeros(E, dtype=np.int32)
@@ -50,7 +55,7 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
         fill = [float(n - nb) for nb in nbar]
     L = x.shape[1]
     slots = [None] * nslots
-    msg_out = np.full((E, L), np.nan)
+    msg_out = np.full((rows, L), np.nan)
     xnew = np.full((n, L), np.nan)
     visited = set()
 
@@ -68,6 +73,12 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
         par, pacc, finp = rec[7], rec[5], rec[6]
         assert par in visited
         acc = take(pacc) + out
+        if sums and rec[9] & 1:            # the wide parent's received sum S_p^t
+            rsum = take(node[par][10]) + out
+            if finp >= 0:
+                msg_out[E + node[par][11]] = rsum
+            else:
+                write(node[par][10], rsum)
         if finp >= 0:
             assert finp == par
             xnew[finp] = acc * scale[finp]
@@ -85,6 +96,7 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
         acc = xh.copy()
         if mode == 1:
             acc = fill[i] * x[i] + xh
+        m_par = np.zeros(L)
         if recv >= 0:
             if flags & 1:
                 # the parent is wide: recv holds its total, which stays live
@@ -92,9 +104,12 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
                 m = slots[recv] - msg_in[pos[pb + ppos][1]]
                 m = 0 * m if lost[pos[pb + ppos][0]] else m
                 msg_out[pos[pb + ppos][0]] = m
-                acc = acc + m
+                m_par = m
             else:
-                acc = acc + take(recv)
+                m_par = take(recv)
+            acc = acc + m_par
+        if sums and deg > REG_DEG:
+            write(rec[10], 0 + m_par)      # S_i^t starts with the DFS parent's message
         if 0 < deg <= REG_DEG:
             m = [msg_in[pos[pb + s][0]] for s in range(deg)]
             for s in range(deg):
@@ -106,7 +121,10 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
                 else:
                     write(pos[pb + s][2], out)
         elif deg > REG_DEG:
-            total = xh + sum(msg_in[pos[pb + s][0]] for s in range(deg))
+            if sums:                       # T_i = x^{t+1/2} + S_i^{t-1}, one row
+                total = xh + msg_in[E + rec[11]]
+            else:
+                total = xh + sum(msg_in[pos[pb + s][0]] for s in range(deg))
             if ppos >= 0:
                 out = total - msg_in[pos[pb + ppos][0]]
                 out = 0 * out if lost[pos[pb + ppos][1]] else out
@@ -122,8 +140,9 @@ def run_program(h, n, x, mu, msg_in, counts_old, lr, sigma, seed, step, mode, c0
     return xnew, msg_out, counts, nslots
 
 
-def check_tree(n, edges, mode, steps=3, L=3, seed=1, p_lost=0.0):
+def check_tree(n, edges, mode, steps=3, L=3, seed=1, p_lost=0.0, sums=False):
     h = rs.relay_create(n, L, edges)
+    rs.relay_set_received_sums(h, sums)
     lost_rng = np.random.default_rng(1000 + n)
     rng = np.random.default_rng(n)
     mu = rng.normal(size=(n, L))
@@ -132,8 +151,10 @@ def check_tree(n, edges, mode, steps=3, L=3, seed=1, p_lost=0.0):
     st = oracle.State(n, edges, L)
     st.x = x.copy()
     st.mu = mu.copy()
-    msg = np.zeros((E, L))
+    msg = np.zeros((rs.relay_message_rows(h), L))
     counts = np.zeros(E, dtype=np.int32)
+    src, dst = rs.relay_edges(h)
+    _, _, node, _ = rs.relay_program(h)
     for t in range(steps):
         lost = (lost_rng.random(E) < p_lost).astype(np.uint8)
         x, msg, counts, nslots = run_program(h, n, x, mu, msg, counts, 0.3, 0.2, seed, t, mode,
@@ -141,42 +162,91 @@ def check_tree(n, edges, mode, steps=3, L=3, seed=1, p_lost=0.0):
         st.advance(1, 0.3, 0.2, seed, mode, drop=lost[None, :] if p_lost > 0 else None)
         assert np.array_equal(counts, st.counts)
         assert np.allclose(x, st.x, rtol=1e-12, atol=1e-12)
-        assert np.allclose(msg, st.msg, rtol=1e-12, atol=1e-12)
+        assert np.allclose(msg[:E], st.msg, rtol=1e-12, atol=1e-12)
+        for i in range(n):  # a sum row holds the sum of the wide node's received messages
+            if node[i][11] >= 0:
+                assert np.allclose(msg[E + node[i][11]], msg[:E][dst == i].sum(axis=0), rtol=1e-12, atol=1e-12)
     return nslots
 
 
+@pytest.mark.parametrize("sums", [False, True])
 @pytest.mark.parametrize("mode", [0, 1])
 @pytest.mark.parametrize("n", [1, 2, 3, 4, 5, 6])
-def test_program_matches_oracle_small_trees(n, mode):
+def test_program_matches_oracle_small_trees(n, mode, sums):
     trees = list(tu.all_trees(n))
     rng = np.random.default_rng(n)
     if len(trees) > 80:
         trees = [trees[k] for k in rng.choice(len(trees), 80, replace=False)]
     for edges in trees:
-        check_tree(n, edges, mode)
+        check_tree(n, edges, mode, sums=sums)
 
 
+def _wide_trees():
+    """Trees with several wide nodes next to each other and next to narrow ones."""
+    # two hubs joined by an edge, each with leaves; a hub whose parent is a hub
+    twin = [(0, 1)] + [(0, k) for k in range(2, 8)] + [(1, k) for k in range(8, 14)]
+    # a chain of three hubs with a narrow node and a subtree between
+    chain3 = ([(0, 1), (1, 2), (2, 3), (3, 4)] + [(0, k) for k in range(5, 10)] +
+              [(2, k) for k in range(10, 15)] + [(4, k) for k in range(15, 21)] + [(15, 21), (21, 22)])
+    return {"twin": np.array(twin, np.int32), "chain3": np.array(chain3, np.int32)}
+
+
+@pytest.mark.parametrize("sums", [False, True])
 @pytest.mark.parametrize("mode", [0, 1])
-@pytest.mark.parametrize("shape", ["star", "chain", "binary", "torus", "random40", "star9"])
-def test_program_matches_oracle_workload_trees(shape, mode):
+@pytest.mark.parametrize("shape", ["star", "chain", "binary", "torus", "random40", "star9", "twin", "chain3"])
+def test_program_matches_oracle_workload_trees(shape, mode, sums):
     trees = {"star": wl.star(64), "chain": wl.chain(64), "binary": wl.binary_tree(64),
              "torus": wl.torus_spanning_tree(8, 8, 0), "random40": wl.random_tree(40, 9),
-             "star9": wl.star(9, hub=4)}
+             "star9": wl.star(9, hub=4), **_wide_trees()}
     edges = trees[shape]
     n = int(edges.max()) + 1
-    check_tree(n, edges, mode, steps=2, L=2)
+    check_tree(n, edges, mode, steps=2 if n > 30 else 5, L=2, sums=sums)
 
 
+@pytest.mark.parametrize("sums", [False, True])
 @pytest.mark.parametrize("mode", [0, 1])
-@pytest.mark.parametrize("shape", ["star", "binary", "random40", "star9", "chain"])
-def test_program_with_lost_messages_matches_oracle(shape, mode):
+@pytest.mark.parametrize("shape", ["star", "binary", "random40", "star9", "chain", "twin", "chain3"])
+def test_program_with_lost_messages_matches_oracle(shape, mode, sums):
     """Lost messages (Section 4.4) are zeroed where the kernel zeroes them --
-    including the messages a wide node's children form from its total."""
+    including the messages a wide node's children form from its total, and
+    the received sums add what arrived."""
     trees = {"star": wl.star(20), "binary": wl.binary_tree(31), "random40": wl.random_tree(40, 9),
-             "star9": wl.star(9, hub=4), "chain": wl.chain(12)}
+             "star9": wl.star(9, hub=4), "chain": wl.chain(12), **_wide_trees()}
     edges = trees[shape]
     n = int(edges.max()) + 1
-    check_tree(n, edges, mode, steps=6, L=2, p_lost=0.25)
+    check_tree(n, edges, mode, steps=6, L=2, p_lost=0.25, sums=sums)
+
+
+def test_received_sums_rows_and_program():
+    """relay_set_received_sums: one sum row per wide node (ascending id), one
+    more slot per wide node, and nothing changes on a tree without one."""
+    star = wl.star(64)
+    h = rs.relay_create(64, 8, star)
+    assert rs.relay_message_rows(h) == 126
+    slots_off = rs.relay_program(h)[0]
+    rs.relay_set_received_sums(h, True)
+    assert rs.relay_message_rows(h) == 127
+    _, _, node, _ = rs.relay_program(h)
+    assert node[0][11] == 0 and node[0][10] >= 0 and (node[1:, 10:] == -1).all()
+    assert rs.relay_program(h)[0] == slots_off + 1
+    rs.relay_set_received_sums(h, False)
+    assert rs.relay_message_rows(h) == 126 and rs.relay_program(h)[0] == slots_off
+    twin = _wide_trees()["chain3"]
+    h = rs.relay_create(23, 8, twin)
+    rs.relay_set_received_sums(h, True)
+    _, _, node, _ = rs.relay_program(h)
+    assert rs.relay_message_rows(h) == 44 + 3
+    assert [int(node[i][11]) for i in (0, 2, 4)] == [0, 1, 2]
+    for tree in (wl.chain(40), wl.binary_tree(40), wl.torus_spanning_tree(8, 8, 0)):
+        n = int(tree.max()) + 1
+        a, b = rs.relay_create(n, 8, tree), rs.relay_create(n, 8, tree)
+        rs.relay_set_received_sums(b, True)
+        assert rs.relay_message_rows(b) == 2 * (n - 1)
+        pa, pb = rs.relay_program(a), rs.relay_program(b)
+        assert pa[0] == pb[0] and np.array_equal(pa[1], pb[1]) and np.array_equal(pa[2], pb[2])
+    lib = ctypes.CDLL(rs.library_path())
+    lib.relay_set_received_sums.argtypes = [ctypes.c_void_p, ctypes.c_int32]
+    assert lib.relay_set_received_sums(h.raw, 2) == rs.RELAY_EINVAL
 
 
 def _rebuild_orders(h, n):
@@ -239,6 +309,13 @@ def test_slot_counts_of_workload_trees():
     assert slots(wl.binary_tree(64)) <= 14
     assert slots(wl.binary_tree(32)) <= 12
     assert slots(wl.star(64)) <= 3
+
+    def slots_with_sums(edges):
+        n = int(edges.max()) + 1
+        h = rs.relay_create(n, 4, edges)
+        rs.relay_set_received_sums(h, True)
+        return rs.relay_program(h)[0]
+    assert slots_with_sums(wl.star(64)) <= 4
     assert slots(wl.torus_spanning_tree(8, 8, 0)) <= 20
 
 
@@ -359,3 +436,31 @@ def test_binding_fails_loudly_without_the_library(monkeypatch, tmp_path):
     monkeypatch.setattr(rs_build, "LIB", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="missing"):
         rs.relay_create(3, 8, wl.chain(3))
+
+
+def test_step_windows_rejects_bad_arguments_before_any_launch():
+    """relay_step_windows checks every window (as relay_step does) and its own
+    arguments on the host before anything is enqueued."""
+    lib = ctypes.CDLL(rs.library_path())
+    vp = ctypes.c_void_p
+    lib.relay_step_windows.argtypes = [vp, ctypes.c_int32, vp, vp, vp, vp, ctypes.c_float, ctypes.c_uint64,
+                                       ctypes.c_int64, vp]
+    a, b = wl.double_binary_trees(8)
+    ha, hb = rs.relay_create(8, 64, a), rs.relay_create(8, 64, b)
+    lib.relay_set_objective.argtypes = [vp, vp, ctypes.c_float]
+    fake = 0x10000
+    big = 1 << 30
+    arr = ctypes.c_void_p * 2
+    hs = arr(ha.raw, hb.raw)
+    xs, mi, mo, cs = arr(fake, fake + 512), arr(big, big + 512), arr(2 * big, 2 * big + 512), arr(fake * 4, fake * 5)
+    # no objective bound on either window
+    assert lib.relay_step_windows(hs, 2, xs, mi, mo, cs, 0.1, 0, 0, None) == rs.RELAY_EINVAL
+    assert lib.relay_set_objective(ha.raw, fake, 0.1) == rs.RELAY_OK
+    assert lib.relay_step_windows(hs, 2, xs, mi, mo, cs, 0.1, 0, 0, None) == rs.RELAY_EINVAL  # window 1
+    assert lib.relay_set_objective(hb.raw, fake, 0.1) == rs.RELAY_OK
+    for count in (0, 3):
+        assert lib.relay_step_windows(hs, count, xs, mi, mo, cs, 0.1, 0, 0, None) == rs.RELAY_EINVAL
+    assert lib.relay_step_windows(arr(ha.raw, ha.raw), 2, xs, mi, mo, cs, 0.1, 0, 0, None) == rs.RELAY_EINVAL
+    assert lib.relay_step_windows(hs, 2, None, mi, mo, cs, 0.1, 0, 0, None) == rs.RELAY_EINVAL
+    assert lib.relay_step_windows(hs, 2, xs, mi, mo, cs, 0.1, 0, -1, None) == rs.RELAY_EINVAL
+    assert lib.relay_step_windows(hs, 2, xs, mi, arr(big, 2 * big), cs, 0.1, 0, 0, None) == rs.RELAY_EINVAL
