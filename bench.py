@@ -298,7 +298,7 @@ def l2_bytes(dev) -> int:
 
 
 def step_bytes(w, args=None) -> int:
-    """HBM bytes one step touches: the algorithmic bytes plus stored centres."""
+    """HBM bytes one step touches: the algorithmic bytes plus the stored mu."""
     stored = args is None or args.objective == "stored"
     return w.bytes_per_step() + (4 * w.d * w.n if stored else 0)
 
@@ -445,17 +445,19 @@ def roofline_of(args, w, run, models_ms) -> dict:
     mean_models_ms = statistics.mean(models_ms)
     state_rows = {"sgd": 0, "nesterov": 2, "adam": 4}[args.optimizer]  # optimiser state read+write
     alg_bytes = w.bytes_per_step() + 4 * w.d * w.n * state_rows
-    moved = alg_bytes if args.objective == "generated" else alg_bytes + 4 * w.d * w.n
+    source = run.objective_source
+    mu_rows = {"stored": w.n, "generated": 0}[source]
+    moved = alg_bytes + 4 * w.d * mu_rows  # the design also reads the stored mu
     achieved = alg_bytes / (mean_models_ms / 1e3) / 1e9
     name = kernel_name_of(run)
     base = name.split(" ")[0]
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4),
-                "traffic": traffic_per_launch(w, args.objective, base, args.optimizer),
+                "traffic": traffic_per_launch(w, source, base, args.optimizer),
                 "kernel": name, "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "algorithmic_bytes_rule": "4 d (2n + 2E) [+ 4 d n x optimiser-state rows]",
-                "objective": args.objective,
+                "objective": source,
                 "design_bytes_per_launch": moved,
                 "achieved_design_bytes": round(moved / (mean_models_ms / 1e3) / 1e9, 1),
                 "launch_ms_mean": round(mean_models_ms, 4),
@@ -590,7 +592,7 @@ def run_fused(args, w, run, dev, stream, world: int) -> dict:
     ms = reduce_max(ev[0].elapsed_time(ev[1]), world)
     fused = all(rs.relay_get_steps_kernel(tr.h) == rs.RELAY_KERNEL_FUSED for tr in run.trees)
     E, state_rows = w.E, {"sgd": 0, "nesterov": 1, "adam": 2}[args.optimizer]
-    mu_rows = w.n if args.objective == "stored" else 0
+    mu_rows = {"stored": w.n, "generated": 0}[run.objective_source]
     # per launch of at most 64 steps: read x, mu, the state, m^{t0-1}; write x, the state and
     # the last two steps' messages
     chunks = -(-K // 64)

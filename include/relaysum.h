@@ -200,25 +200,6 @@ int relay_set_objective(relay_handle *h, const float *mu, float sigma);
 int relay_set_objective_generated(relay_handle *h, const float *mix, int32_t K, float mu_scale,
                                   uint64_t mu_seed, float sigma);
 
-/* Writes the K Gaussian centres N_1 .. N_K themselves (Philox stream 1, row
- * k, at the handle's coordinate offset) to `centres`, a device fp32 [K][ld]
- * array (stride ld_x); the columns [d, 4 ceil(d/4)) are zeroed. */
-int relay_fill_centres(relay_handle *h, float *centres, int32_t K, uint64_t mu_seed, relay_stream_t stream);
-
-/* Binds the same objective with mu formed in the kernel from K stored
- * Gaussian centres: `centres` is a caller-owned device fp32 [K][ld] array
- * holding N_1 .. N_K (as relay_fill_centres writes them; read, never
- * written), `mix` a HOST
- * fp32 [n][K] matrix whose non-zeros are copied into the handle.  mu_i =
- * mu_scale * sum_k mix[i][k] N_k is formed in fp32 in the order
- * relay_fill_objective uses, so every result equals that of the stored mu
- * bit for bit, while a step reads K centre rows instead of n rows of mu --
- * fewer bytes when K < n (a mixture of few centres, such as the Dirichlet
- * mixtures of the heterogeneity experiments).  RELAY_EUNSUPPORTED if K > 16
- * or mix has more than 1024 non-zeros. */
-int relay_set_objective_centres(relay_handle *h, const float *centres, const float *mix, int32_t K,
-                                float mu_scale, float sigma);
-
 /* Fills mu (device fp32 [n][ld]) with mu_i(c) = mu_scale * sum_k
  * mix[i][k] N_k(c): K Gaussian centres N_k (Philox stream 1, row k) mixed by
  * the device fp32 [n][K] matrix `mix` (identity for one centre per worker,
@@ -318,8 +299,8 @@ int relay_steps(relay_handle *h, float *x, float *msg_a, float *msg_b, int32_t *
  * evolves on its own and the noise is keyed by the absolute coordinate, so
  * the result equals relay_step on the resident state bit for bit.  The
  * handle must use regenerated centres (relay_set_objective_generated) and
- * the SGD local step: a device mu or centres array, or optimiser state, has
- * no place in a host-state step (RELAY_EUNSUPPORTED otherwise).
+ * the SGD local step: a device mu array or optimiser state has no place in
+ * a host-state step (RELAY_EUNSUPPORTED otherwise).
  *
  * Copies: only the message rows a step reads go in -- every row except
  * those arriving at a leaf, whose one outgoing message excludes its one
@@ -367,7 +348,7 @@ int relay_host_bytes(const relay_host_plan *p, int64_t *h2d, int64_t *d2h);
  * m^{t-1}, msg_out <- m^t, counts c^{t-1} -> c^t, all page-locked host
  * arrays; lr, seed and step as relay_step.  Errors: RELAY_EINVAL (NULL or
  * pageable host array, another device than the plan's, step out of range,
- * no objective), RELAY_EUNSUPPORTED (stored centres or an optimiser with
+ * no objective), RELAY_EUNSUPPORTED (a stored mu or an optimiser with
  * state), RELAY_ECUDA. */
 int relay_step_host(relay_host_plan *p, float *x, const float *msg_in, float *msg_out, int32_t *counts,
                     float lr, uint64_t seed, int64_t step, relay_stream_t stream);

@@ -25,8 +25,7 @@ from ._native import (RELAY_EINVAL, RELAY_ECUDA, RELAY_ENOMEM, RELAY_ENOTTREE, R
                       relay_metrics_static, relay_metrics_workspace, relay_nbar, relay_num_edges,
                       relay_program, relay_set_coord_offset, relay_set_objective,
                       relay_set_algorithm, relay_set_local_optimizer, relay_set_lost_messages,
-                      relay_set_objective_generated, relay_set_objective_centres, relay_fill_centres,
-                      relay_get_kernel,
+                      relay_set_objective_generated, relay_get_kernel,
                       relay_get_steps_kernel,
                       relay_set_kernel, relay_set_rebuild_mode, relay_set_strides,
                       relay_set_received_sums, relay_message_rows, relay_step, relay_step_windows,
@@ -45,7 +44,7 @@ __all__ = [
     "relay_set_rebuild_mode", "relay_set_kernel", "relay_get_kernel", "relay_get_steps_kernel",
     "relay_set_strides", "relay_set_local_optimizer", "relay_set_received_sums", "relay_message_rows",
     "relay_set_lost_messages", "relay_set_algorithm", "relay_set_coord_offset", "relay_set_objective",
-    "relay_set_objective_generated", "relay_set_objective_centres", "relay_fill_centres", "relay_fill_objective", "relay_init", "relay_step_counts",
+    "relay_set_objective_generated", "relay_fill_objective", "relay_init", "relay_step_counts",
     "relay_step_models", "relay_step", "relay_step_windows", "relay_steps",
     "relay_nbar", "relay_program", "relay_metrics", "relay_metrics_workspace",
     "relay_metrics_static",

@@ -133,8 +133,7 @@ int check_host_args(relay_host_plan* p, const float* x, const float* msg_in, con
     const relay_handle* h = p->h;
     if (!h->has_objective || !std::isfinite(lr)) return RELAY_EINVAL;
     // device-resident inputs have no place in a host-state step
-    if (h->obj.source == relaysum::kMuStored || h->obj.source == relaysum::kMuStoredCentres || h->opt != RELAY_OPT_SGD)
-        return RELAY_EUNSUPPORTED;
+    if (h->obj.source == relaysum::kMuStored || h->opt != RELAY_OPT_SGD) return RELAY_EUNSUPPORTED;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev != p->dev) return RELAY_EINVAL;
     if (p->E > 0 && !counts) return RELAY_EINVAL;

@@ -95,7 +95,6 @@ enum ObjectiveSource : int32_t {
     kMuStored = 0,      // read the caller's mu array
     kMuPerRow = 1,      // regenerate: one Philox block per non-zero weight of the row
     kMuCachedCentres = 2,  // regenerate the K centres once per quad, then mix per row
-    kMuStoredCentres = 3,  // read the caller's K centres once per quad, then mix per row
 };
 
 struct Objective {

@@ -432,26 +432,18 @@ __device__ __forceinline__ float4 local_update(const ModelArgs& a, int i, int64_
     return u;
 }
 
-// mu_i for quad q: read, or formed from the K Gaussian centres exactly as
-// relay_fill_mu_kernel writes it (the same normals, the same fma order), so
-// every source gives the same bits.  The centres are regenerated
-// (kMuPerRow, kMuCachedCentres) or read from the caller's [K][ld_x] array
-// (kMuStoredCentres, a.mu); `cen` holds the quad's K centres in shared
-// memory where the walk cached them, else null.
+// mu_i for quad q: read, or regenerated exactly as relay_fill_mu_kernel
+// writes it (same normals, same fma order), so both sources give the same bits.
 template <int OBJ>
 __device__ __forceinline__ float4 centre(const Objective& obj, const PhiloxKey& mu_key, const ModelArgs& a,
                                          int i, int64_t q, const float4* cen, int cen_stride) {
     if (OBJ == relaysum::kMuStored) return ld_stream(a.mu + i * a.ld_x + 4 * q);
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int j = obj.row_off[i]; j < obj.row_off[i + 1]; ++j) {
-        float4 z;
-        if (OBJ == relaysum::kMuPerRow) {
-            z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(obj.col[j]), 0u, 1u, mu_key);
-        } else if (OBJ == relaysum::kMuStoredCentres && cen == nullptr) {
-            z = ld_stream(a.mu + obj.col[j] * a.ld_x + 4 * q);
-        } else {
-            z = cen[obj.col[j] * cen_stride];
-        }
+        const float4 z = (OBJ == relaysum::kMuPerRow)
+                             ? normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(obj.col[j]),
+                                       0u, 1u, mu_key)
+                             : cen[obj.col[j] * cen_stride];
         acc = fma4(obj.w[j], z, acc);
     }
     return scale4_rn(acc, obj.scale);
@@ -542,17 +534,13 @@ relay_models_kernel(const __grid_constant__ Windows<NT> win, const __grid_consta
     rebuild_factors(prog, a, s_scale, s_fill);
     __syncthreads();
     const Slots sl{slot_mem + threadIdx.x, static_cast<int>(blockDim.x)};
-    // the quad's K centres, regenerated or read once per quad (kMuCachedCentres, kMuStoredCentres)
-    float4* cen = slot_mem + prog.nslots * blockDim.x + threadIdx.x;
+    float4* cen = slot_mem + prog.nslots * blockDim.x + threadIdx.x;  // OBJ == kMuCachedCentres
     const int64_t stride = ctas * blockDim.x;
     for (int64_t q = cta * blockDim.x + threadIdx.x; q < a.nquads; q += stride) {
         if (OBJ == relaysum::kMuCachedCentres) {
             for (int k = 0; k < obj.K; ++k)
                 cen[k * blockDim.x] = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k), 0u,
                                               1u, mu_key);
-        }
-        if (OBJ == relaysum::kMuStoredCentres) {
-            for (int k = 0; k < obj.K; ++k) cen[k * blockDim.x] = ld_stream(a.mu + k * a.ld_x + 4 * q);
         }
         // x (and a stored mu) of the next node in the walk are loaded one visit
         // early, so their latency overlaps the current visit's arithmetic
@@ -694,9 +682,8 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
     __shared__ float s_scale[kMaxN];
     __shared__ float s_fill[kMaxN];
     // regenerated centres are formed per row (the walk's cached centres are
-    // the same normals mixed in the same order); stored centres are read per
-    // non-zero of the row
-    constexpr int kObj = (OBJ == relaysum::kMuCachedCentres) ? relaysum::kMuPerRow : OBJ;
+    // the same normals mixed in the same order)
+    constexpr int kObj = (OBJ == relaysum::kMuStored) ? relaysum::kMuStored : relaysum::kMuPerRow;
     const int i = static_cast<int>(threadIdx.x) / qb;
     const int qi = static_cast<int>(threadIdx.x) - i * qb;
     float4* const buf0 = node_mem + qi;                     // [e * qb]: m^t on edge e (even blocks)
@@ -851,7 +838,7 @@ relay_fused_steps_kernel(const __grid_constant__ Program prog, const __grid_cons
                          const __grid_constant__ FusedSteps fs, int qb) {
     extern __shared__ float4 fused_mem[];
     __shared__ int32_t c_mem[2][kMaxE];  // counters of the step parities
-    constexpr int kObj = (OBJ == relaysum::kMuCachedCentres) ? relaysum::kMuPerRow : OBJ;
+    constexpr int kObj = (OBJ == relaysum::kMuStored) ? relaysum::kMuStored : relaysum::kMuPerRow;
     const int tid = static_cast<int>(threadIdx.x);
     const int i = tid / qb;
     const int qi = tid - i * qb;
@@ -983,21 +970,6 @@ __global__ void relay_fill_mu_kernel(float* mu, const float* mix, int n, int K, 
             const float4 sv = scale4_rn(acc, scale);
             *reinterpret_cast<float4*>(mu + i * ld_x + c) =
                 make_float4(sv.x, c + 1 < d ? sv.y : 0.f, c + 2 < d ? sv.z : 0.f, c + 3 < d ? sv.w : 0.f);
-        }
-    }
-}
-
-// The K Gaussian centres N_k themselves ([K][ld_x], Philox stream 1, row k),
-// as relay_fill_mu_kernel draws them; ragged columns beyond d are zero.
-__global__ void relay_fill_centres_kernel(float* centres, int K, int64_t ld_x, int64_t nquads, int64_t d,
-                                          uint32_t q0, const __grid_constant__ PhiloxKey key) {
-    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < nquads; q += stride) {
-        const int64_t c = 4 * q;
-        for (int k = 0; k < K; ++k) {
-            const float4 z = normal4(q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(k), 0u, 1u, key);
-            *reinterpret_cast<float4*>(centres + k * ld_x + c) =
-                make_float4(z.x, c + 1 < d ? z.y : 0.f, c + 2 < d ? z.z : 0.f, c + 3 < d ? z.w : 0.f);
         }
     }
 }
@@ -1200,8 +1172,7 @@ int launch_models(const relay_handle* const* hs, const ModelArgs* as, cudaStream
     if (sms <= 0) return RELAY_ECUDA;
     int per_thread = 0;
     for (int k = 0; k < NT; ++k)
-        per_thread = std::max(per_thread, hs[k]->prog.nslots + (OBJ == relaysum::kMuCachedCentres ||
-                                                                OBJ == relaysum::kMuStoredCentres ? hs[k]->obj.K : 0));
+        per_thread = std::max(per_thread, hs[k]->prog.nslots + (OBJ == relaysum::kMuCachedCentres ? hs[k]->obj.K : 0));
     const int threads = models_threads(per_thread);
     const size_t smem = static_cast<size_t>(per_thread) * threads * 16;
     if (smem > static_cast<size_t>(kMaxSmem)) return RELAY_EUNSUPPORTED;
@@ -1285,8 +1256,6 @@ int launch_walk_src(const relay_handle* const* hs, const ModelArgs* as, cudaStre
     switch (hs[0]->obj.source) {
         case relaysum::kMuStored: return launch_models<relaysum::kMuStored, OPT, NT, WIDE>(hs, as, stream, after_counts);
         case relaysum::kMuPerRow: return launch_models<relaysum::kMuPerRow, OPT, NT, WIDE>(hs, as, stream, after_counts);
-        case relaysum::kMuStoredCentres:
-            return launch_models<relaysum::kMuStoredCentres, OPT, NT, WIDE>(hs, as, stream, after_counts);
         default: return launch_models<relaysum::kMuCachedCentres, OPT, NT, WIDE>(hs, as, stream, after_counts);
     }
 }
@@ -1304,8 +1273,6 @@ int launch_models_obj(const relay_handle* h, const ModelArgs& a, cudaStream_t st
     if (use_nodes(h)) {
         if (h->obj.source == relaysum::kMuStored)
             return launch_nodes<relaysum::kMuStored, OPT>(h, a, stream, after_counts);
-        if (h->obj.source == relaysum::kMuStoredCentres)
-            return launch_nodes<relaysum::kMuStoredCentres, OPT>(h, a, stream, after_counts);
         return launch_nodes<relaysum::kMuPerRow, OPT>(h, a, stream, after_counts);
     }
     return launch_walk_obj<OPT, 1>(&h, &a, stream, after_counts);
@@ -1358,8 +1325,6 @@ bool use_fused(const relay_handle* h) {
 template <int OPT>
 int launch_fused_obj(const relay_handle* h, const ModelArgs& a, const FusedSteps& fs, cudaStream_t stream) {
     if (h->obj.source == relaysum::kMuStored) return launch_fused<relaysum::kMuStored, OPT>(h, a, fs, stream);
-    if (h->obj.source == relaysum::kMuStoredCentres)
-        return launch_fused<relaysum::kMuStoredCentres, OPT>(h, a, fs, stream);
     return launch_fused<relaysum::kMuPerRow, OPT>(h, a, fs, stream);
 }
 
@@ -1613,24 +1578,6 @@ int relay_set_objective_generated(relay_handle* h, const float* mix, int32_t K, 
     return RELAY_OK;
 }
 
-int relay_set_objective_centres(relay_handle* h, const float* centres, const float* mix, int32_t K,
-                                float mu_scale, float sigma) {
-    if (!h || K < 1 || !mix || !std::isfinite(mu_scale) || !std::isfinite(sigma) || sigma < 0.0f)
-        return RELAY_EINVAL;
-    if (h->d > 0 && (!centres || !aligned16(centres))) return RELAY_EINVAL;
-    if (K > relaysum::kMaxCachedCentres) return RELAY_EUNSUPPORTED;
-    Objective o;
-    int nnz = 0;
-    const int rc = mixture(h, mix, K, mu_scale, &o, &nnz);
-    if (rc != RELAY_OK) return rc;
-    o.source = relaysum::kMuStoredCentres;
-    h->obj = o;
-    h->mu = centres;
-    h->sigma = sigma;
-    h->has_objective = true;
-    return RELAY_OK;
-}
-
 int relay_fill_objective(relay_handle* h, float* mu, const float* mix, int32_t K, float mu_scale,
                          uint64_t mu_seed, relay_stream_t stream) {
     if (!h || K < 0 || !std::isfinite(mu_scale)) return RELAY_EINVAL;
@@ -1640,16 +1587,6 @@ int relay_fill_objective(relay_handle* h, float* mu, const float* mix, int32_t K
     relay_fill_mu_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
         mu, mix, h->prog.n, K, h->ld_x, h->nquads, h->d, static_cast<uint32_t>(h->c0 / 4), mu_scale,
         philox_key(mu_seed));
-    return launch_status();
-}
-
-int relay_fill_centres(relay_handle* h, float* centres, int32_t K, uint64_t mu_seed, relay_stream_t stream) {
-    if (!h || K < 1) return RELAY_EINVAL;
-    if (h->d == 0) return RELAY_OK;
-    if (!centres || !aligned16(centres)) return RELAY_EINVAL;
-    const int threads = 256;
-    relay_fill_centres_kernel<<<grid_for(h->nquads, threads), threads, 0, stream>>>(
-        centres, K, h->ld_x, h->nquads, h->d, static_cast<uint32_t>(h->c0 / 4), philox_key(mu_seed));
     return launch_status();
 }
 
@@ -1925,10 +1862,6 @@ int relay_metrics(relay_handle* h, const float* x, double* workspace, double* ou
     switch (h->obj.source) {
         case relaysum::kMuStored:
             relay_metrics_kernel<relaysum::kMuStored><<<blocks, kMetricsThreads, 0, stream>>>(
-                h->obj, mu_key, a, n, h->d, workspace);
-            break;
-        case relaysum::kMuStoredCentres:
-            relay_metrics_kernel<relaysum::kMuStoredCentres><<<blocks, kMetricsThreads, 0, stream>>>(
                 h->obj, mu_key, a, n, h->d, workspace);
             break;
         default:  // cached centres are regenerated per row here

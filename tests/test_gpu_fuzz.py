@@ -62,7 +62,7 @@ def draw(case: int) -> dict:
                 lr=float(rng.uniform(0.01, 0.3)), sigma=float(rng.uniform(0.0, 0.3)),
                 x0_std=float(rng.choice([0.0, 0.5])), mu_scale=float(rng.uniform(0.5, 3.0)),
                 seed=int(rng.integers(0, 2**40)), mu_seed=int(rng.integers(0, 2**40)),
-                # drawn from a stream of its own, so the other draws of each case are unchanged
+                # drawn from streams of their own, so the other draws of each case are unchanged
                 received_sums=bool(np.random.default_rng(5000 + case).integers(0, 2)))
 
 
@@ -72,8 +72,9 @@ def test_random_configuration_against_oracle(case):
     n, d, E = c["n"], c["d"], 2 * (c["n"] - 1)
     optimizer = {"sgd": None, "nesterov": ("nesterov", c["beta1"]),
                  "adam": ("adam", c["beta1"], c["beta2"], 1e-2)}[c["opt"]]
+    objective = c["objective"]
     run = rs.RelayRun(n, d, c["edges"], device="cuda:0", mode=c["mode"], c0=c["c0"],
-                      objective=c["objective"], optimizer=optimizer, algorithm=c["algo"], kernel=c["kernel"],
+                      objective=objective, optimizer=optimizer, algorithm=c["algo"], kernel=c["kernel"],
                       received_sums=c["received_sums"])
     run.init(c["x0_std"], c["seed"], c["mix"], c["mu_scale"], c["mu_seed"], c["sigma"])
     st = oracle.State(n, c["edges"], d, c0=c["c0"])

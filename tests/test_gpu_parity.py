@@ -276,8 +276,7 @@ def test_full_size_workload_sampled(w):
 
 def test_double16_full_size_sampled():
     """Double binary trees (Section 3) at the VGG-11 size, 200 steps, as
-    bench.py runs them (stored centres, both windows in one relay_step_windows
-    launch).
+    bench.py runs them (stored centres, the two windows on forked streams).
     In each tree's coordinate window the oracle runs that tree on the first
     and last 65,536 coordinates and 1,024 random windows of 1,024."""
     _free()
@@ -321,10 +320,10 @@ def test_binary16_resnet20_every_coordinate_mode0():
     assert np.array_equal(run.counts.cpu().numpy(), st.counts)
 
 
-def test_double_tree_steps_in_graphs_and_eagerly():
-    """Double binary trees: RelayRun.step runs both tree windows in one
-    relay_step_windows call; the eager run, a CUDA graph of the same steps
-    replayed once, and relay_step issued window by window agree bit for bit."""
+def test_double_tree_steps_fork_and_join_in_graphs_and_eagerly():
+    """Double binary trees: RelayRun.step runs the two tree windows on forked
+    streams; the eager run, a CUDA graph of the same steps replayed once,
+    and steps issued window by window on one stream agree bit for bit."""
     n, d = 16, 40_001
     trees = list(wl.double_binary_trees(n))
     runs = []
