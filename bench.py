@@ -352,7 +352,8 @@ def make_run(args, w, dev, c0: int):
 def make_stepper(args, w, run, stream, rank: int):
     """one_step(ev): one step of `run` on `stream`; ev (per tree window: three
     CUDA events) brackets the counter kernel and the step kernel.  Several
-    tree windows (double binary trees) are one step, timed as a whole."""
+    tree windows (double binary trees) are one relay_step_windows call (one
+    counter launch, one step-kernel launch), timed as a whole."""
     import numpy as np
     import torch
 
@@ -432,7 +433,7 @@ def kernel_name_of(run) -> str:
     name = ("relay_nodes_kernel" if rs.relay_get_kernel(run.h) == rs.RELAY_KERNEL_NODES
             else "relay_models_kernel")
     T = len(run.trees)
-    return name if T == 1 else f"{name} on {T} tree windows, overlapped (whole step timed)"
+    return name if T == 1 else f"{name} over {T} tree windows in one launch (relay_step_windows; whole step timed)"
 
 
 def roofline_of(args, w, run, models_ms) -> dict:

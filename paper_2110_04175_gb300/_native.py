@@ -418,9 +418,8 @@ class RelayRun:
     two message buffers [rows][ld_tree] (double buffering; rows = E plus the
     wide nodes' received sums) and counters int32 [E], and -- for
     objective="stored" -- the centres mu [n][ld] (objective="generated" lets
-    the kernel regenerate them).  ``step()`` enqueues one relay_step per tree
-    on the current torch stream (several trees on forked streams);
-    ``step_windows()`` steps all trees with one relay_step_windows call.
+    the kernel regenerate them).  ``step()`` enqueues one step on the current
+    torch stream: relay_step, or relay_step_windows for several trees.
     """
 
     def __init__(self, n: int, d: int, edges, device="cuda", mode: int = 1, c0: int = 0,
@@ -620,26 +619,30 @@ class RelayRun:
             main.wait_event(done)
 
     def step(self, lr: float, seed: int, stream=None):
-        """Enqueues one step (relay_step per tree) on `stream`; several tree
-        windows run on forked streams (_per_tree), which measured 1.4 % faster
-        on the double binary trees than their one-launch relay_step_windows
-        (step_windows)."""
+        """Enqueues one step on `stream` (default: the current stream): relay_step,
+        or with several tree windows one relay_step_windows call (one counter
+        launch and one step-kernel launch for the windows where they allow it;
+        it measured the same as the windows on forked streams, step_forked)."""
+        trs = self.trees
+        if len(trs) == 1:
+            tr = trs[0]
+            relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed, self.t, stream)
+        else:
+            relay_step_windows([tr.h for tr in trs], [self._x(tr) for tr in trs], [tr.msg[tr.cur] for tr in trs],
+                               [tr.msg[1 - tr.cur] for tr in trs], [tr.counts for tr in trs], lr, seed, self.t,
+                               stream)
+        for tr in trs:
+            tr.cur = 1 - tr.cur
+        self.t += 1
+
+    def step_forked(self, lr: float, seed: int, stream=None):
+        """The same step with one relay_step per tree window, the windows on
+        streams forked from `stream` and joined back (the same bits as step())."""
         def issue(tr, s):
             relay_step(tr.h, self._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed, self.t, s)
             tr.cur = 1 - tr.cur
 
         self._per_tree(issue, stream)
-        self.t += 1
-
-    def step_windows(self, lr: float, seed: int, stream=None):
-        """Enqueues one step of every tree window with one relay_step_windows
-        call on `stream`: one counter launch and one step-kernel launch for the
-        windows where they allow it.  The same bits as step()."""
-        trs = self.trees
-        relay_step_windows([tr.h for tr in trs], [self._x(tr) for tr in trs], [tr.msg[tr.cur] for tr in trs],
-                           [tr.msg[1 - tr.cur] for tr in trs], [tr.counts for tr in trs], lr, seed, self.t, stream)
-        for tr in trs:
-            tr.cur = 1 - tr.cur
         self.t += 1
 
     def steps(self, k: int, lr: float, seed: int, stream=None):

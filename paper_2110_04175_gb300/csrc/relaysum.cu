@@ -513,22 +513,16 @@ struct Windows {
     int32_t split;
 };
 
-// OBJ: where mu comes from (ObjectiveSource).  OPT: the local optimiser
-// (0 SGD, 1 Nesterov momentum, 2 Adam).  NT: windows per launch.  WIDE: some
-// node has more than kRegDeg neighbours; without one the wide-node paths are
-// not compiled, and they cost the narrow trees nothing.
-template <int OBJ, int OPT, int NT, bool WIDE>
-__global__ void __launch_bounds__(128)
-relay_models_kernel(const __grid_constant__ Windows<NT> win, const __grid_constant__ Objective obj,
-                    const __grid_constant__ PhiloxKey mu_key) {
-    extern __shared__ float4 slot_mem[];
-    __shared__ float s_scale[kMaxN];
-    __shared__ float s_fill[kMaxN];
-    const int wdw = (NT == 1) ? 0 : (static_cast<int>(blockIdx.x) >= win.split ? 1 : 0);
-    const Program& prog = win.prog[wdw];
-    const ModelArgs& a = win.a[wdw];
-    const int64_t cta = (NT == 1) ? blockIdx.x : static_cast<int64_t>(blockIdx.x) - (wdw ? win.split : 0);
-    const int64_t ctas = (NT == 1) ? gridDim.x : (wdw ? static_cast<int64_t>(gridDim.x) - win.split : win.split);
+// The walk over one window's quads: CTA `cta` of `ctas` takes quads
+// cta*blockDim + threadIdx, stepping by ctas*blockDim.  OBJ: where mu comes
+// from (ObjectiveSource).  OPT: the local optimiser (0 SGD, 1 Nesterov
+// momentum, 2 Adam).  WIDE: some node has more than kRegDeg neighbours;
+// without one the wide-node paths are not compiled, and they cost the narrow
+// trees nothing.
+template <int OBJ, int OPT, bool WIDE>
+__device__ __forceinline__ void walk(const Program& prog, const ModelArgs& a, const Objective& obj,
+                                     const PhiloxKey& mu_key, int64_t cta, int64_t ctas, float4* slot_mem,
+                                     float* s_scale, float* s_fill) {
     const int n = prog.n;
     wait_for_prior_grid();
     rebuild_factors(prog, a, s_scale, s_fill);
@@ -602,6 +596,27 @@ relay_models_kernel(const __grid_constant__ Windows<NT> win, const __grid_consta
                 sl[r.acc_slot] = acc;
             }
         }
+    }
+}
+
+// The step kernel over NT windows.  The walk is inlined once per window, so
+// each copy reads its window's program and arguments at fixed parameter
+// offsets (constant operands), as the one-window kernel does; the grid's
+// first `split` CTAs take window 0.
+template <int OBJ, int OPT, int NT, bool WIDE>
+__global__ void __launch_bounds__(128)
+relay_models_kernel(const __grid_constant__ Windows<NT> win, const __grid_constant__ Objective obj,
+                    const __grid_constant__ PhiloxKey mu_key) {
+    extern __shared__ float4 slot_mem[];
+    __shared__ float s_scale[kMaxN];
+    __shared__ float s_fill[kMaxN];
+    if (NT == 1) {
+        walk<OBJ, OPT, WIDE>(win.prog[0], win.a[0], obj, mu_key, blockIdx.x, gridDim.x, slot_mem, s_scale, s_fill);
+    } else if (static_cast<int>(blockIdx.x) < win.split) {
+        walk<OBJ, OPT, WIDE>(win.prog[0], win.a[0], obj, mu_key, blockIdx.x, win.split, slot_mem, s_scale, s_fill);
+    } else {
+        walk<OBJ, OPT, WIDE>(win.prog[NT - 1], win.a[NT - 1], obj, mu_key, blockIdx.x - win.split,
+                             gridDim.x - win.split, slot_mem, s_scale, s_fill);
     }
 }
 

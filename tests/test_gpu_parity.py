@@ -276,7 +276,8 @@ def test_full_size_workload_sampled(w):
 
 def test_double16_full_size_sampled():
     """Double binary trees (Section 3) at the VGG-11 size, 200 steps, as
-    bench.py runs them (stored centres, the two windows on forked streams).
+    bench.py runs them (stored centres, both windows in one relay_step_windows
+    launch).
     In each tree's coordinate window the oracle runs that tree on the first
     and last 65,536 coordinates and 1,024 random windows of 1,024."""
     _free()
@@ -320,20 +321,22 @@ def test_binary16_resnet20_every_coordinate_mode0():
     assert np.array_equal(run.counts.cpu().numpy(), st.counts)
 
 
-def test_double_tree_steps_fork_and_join_in_graphs_and_eagerly():
-    """Double binary trees: RelayRun.step runs the two tree windows on forked
-    streams; the eager run, a CUDA graph of the same steps replayed once,
-    and steps issued window by window on one stream agree bit for bit."""
+def test_double_tree_steps_in_graphs_and_eagerly():
+    """Double binary trees: RelayRun.step runs both tree windows in one
+    relay_step_windows call, step_forked on forked streams; the eager run,
+    a CUDA graph of the same steps replayed once, a forked run and relay_step
+    issued window by window on one stream agree bit for bit."""
     n, d = 16, 40_001
     trees = list(wl.double_binary_trees(n))
     runs = []
-    for _ in range(3):
-        r = rs.RelayRun(n, d, trees, device="cuda:0")
+    for _ in range(4):
+        r = rs.RelayRun(n, d, trees, device="cuda:0", kernel="walk")
         r.init(0.1, 3, wl.identity_mix(n), 1.0, 4, 0.1)
         runs.append(r)
-    eager, graphed, serial = runs
+    eager, graphed, serial, forked = runs
     for _ in range(25):
         eager.step(0.05, 3)
+        forked.step_forked(0.05, 3)
     for _ in range(5):
         graphed.step(0.05, 3)
     g = graphed.capture(20, 0.05, 3)
@@ -343,7 +346,7 @@ def test_double_tree_steps_fork_and_join_in_graphs_and_eagerly():
             rs.relay_step(tr.h, serial._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, 0.05, 3, t)
             tr.cur = 1 - tr.cur
     torch.cuda.synchronize()
-    for other in (graphed, serial):
+    for other in (graphed, serial, forked):
         assert torch.equal(other.x[:, :d], eager.x[:, :d])
         for ta, tb in zip(other.trees, eager.trees):
             assert torch.equal(ta.messages[:ta.E, :ta.d], tb.messages[:tb.E, :tb.d])

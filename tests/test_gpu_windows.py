@@ -87,7 +87,7 @@ def test_step_windows_equals_relay_step_per_window(name):
                 lost = (rng.random(tr.E) < c["lost_p"]).astype(np.uint8)
                 a.set_lost(lost, tree=k)
                 b.set_lost(lost, tree=k)
-        a.step_windows(lr, seed)
+        a.step(lr, seed)  # relay_step_windows
         for tr in b.trees:
             rs.relay_step(tr.h, b._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, lr, seed, b.t)
             tr.cur = 1 - tr.cur
@@ -112,7 +112,7 @@ def test_windows_with_different_objectives_fall_back():
         runs.append(r)
     a, b = runs
     for _ in range(6):
-        a.step_windows(0.05, 2)
+        a.step(0.05, 2)
         for tr in b.trees:
             rs.relay_step(tr.h, b._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts, 0.05, 2, b.t)
             tr.cur = 1 - tr.cur
@@ -129,7 +129,7 @@ def test_one_launch_windows_match_two_oracle_runs():
     run = rs.RelayRun(n, d, [a, b], device="cuda:0", kernel="walk")
     run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
     for _ in range(steps):
-        run.step_windows(w.lr, w.seed)
+        run.step(w.lr, w.seed)
     torch.cuda.synchronize()
     for tr, edges in zip(run.trees, (a, b)):
         wt = wl.Workload("dbt", n, edges, d, w.mix, 1.0, 0.05, 0.05, 0.1, steps)
@@ -142,16 +142,17 @@ def test_one_launch_windows_match_two_oracle_runs():
 def test_double16_full_size_one_launch_equals_forked_streams():
     """The VGG-11-sized double binary trees, 200 steps, in the launch
     configuration of the bench (stored centres, the automatic kernel: the
-    walk): relay_step_windows equals the two windows on forked streams (whose
-    full-size parity against the oracle test_gpu_parity checks), bit for bit,
-    where each CTA of the one launch loops over many quads of its window."""
+    walk): relay_step_windows (whose full-size parity against the oracle
+    test_gpu_parity checks) equals the two windows stepped by relay_step on
+    forked streams, bit for bit, where each CTA of the one launch loops over
+    many quads of its window."""
     w = wl.double16_vgg11()
     states = []
     for one_launch in (True, False):
         run = rs.RelayRun(w.n, w.d, w.edges, device="cuda:0", mode=w.mode)
         run.init(w.x0_std, w.seed, w.mix, w.mu_scale, w.mu_seed, w.sigma)
         for _ in range(w.steps):
-            (run.step_windows if one_launch else run.step)(w.lr, w.seed)
+            (run.step if one_launch else run.step_forked)(w.lr, w.seed)
         torch.cuda.synchronize()
         states.append([t.cpu() for t in _state(run)])
         del run
