@@ -19,8 +19,10 @@ on every host core (one slice per thread) and on one thread.
 
 Multi-GPU (torchrun, one rank per GPU): every rank runs the same workload on
 its own d-slice of one longer model vector (coordinates are independent, so
-there is no data-path collective; weak scaling).  `--impl reference` times
-the CPU oracle instead (rank 0 only).
+there is no data-path collective; weak scaling).  With more local ranks than
+visible GPUs the ranks share them round robin and the process group uses
+gloo (a functional check of the multi-rank path; such a line is no scaling
+figure).  `--impl reference` times the CPU oracle instead (rank 0 only).
 """
 from __future__ import annotations
 
@@ -66,6 +68,21 @@ def reduce_max(value: float, world: int) -> float:
 def reduce_min(value: float, world: int) -> float:
     """Min over ranks (used for decisions every rank must take alike)."""
     return -reduce_max(-value, world)
+
+
+def local_device(local: int, n_devices: int) -> int:
+    """The GPU of local rank `local`: its own where every local rank has one,
+    else round robin over the visible GPUs (the ranks then share them)."""
+    if n_devices <= 0:
+        raise RuntimeError("bench.py's native arm needs a CUDA device")
+    return local % n_devices
+
+
+def process_group_backend(local_world: int, n_devices: int) -> str:
+    """NCCL where every local rank has a GPU of its own; gloo (host
+    collectives) where ranks share one, which NCCL refuses.  The path has no
+    data-path collective, only the barrier and the max over ranks."""
+    return "nccl" if local_world <= n_devices else "gloo"
 
 
 def barrier(world: int):
@@ -320,6 +337,21 @@ def l2_note(w, args, dev=None) -> str:
     return f"inputs larger than L2 ({mb / 1e3:.1f} GB moved per step)"
 
 
+def parallelism_note(gpus: int) -> str:
+    if gpus <= 1:
+        return "1 GPU"
+    note = f"d-sharded over {gpus} rank(s), no collective"
+    try:
+        import torch
+        n_dev = torch.cuda.device_count()
+    except Exception:  # noqa: BLE001 - the note is informational
+        return note
+    local_world = int(os.environ.get("LOCAL_WORLD_SIZE", str(gpus)))
+    if 0 < n_dev < local_world:
+        note += f"; {local_world} local ranks share {n_dev} GPU(s) (functional check, not a scaling figure)"
+    return note
+
+
 def workload_config(w, gpus: int, args=None, dev=None) -> dict:
     shape = {"binary": "balanced binary tree (heap order)", "chain": "chain", "star": "star",
              "torus": "uniform spanning tree of the 8x8 torus",
@@ -329,8 +361,7 @@ def workload_config(w, gpus: int, args=None, dev=None) -> dict:
             "rebuild": "robust (Section 4.4)" if w.mode == 1 else "Algorithm 1",
             "sigma": w.sigma, "lr": w.lr, "objective": "identity-Hessian heterogeneous quadratics",
             "l2": l2_note(w, args, dev),
-            "parallelism": f"d-sharded over {gpus} rank(s), no collective" if gpus > 1
-            else "1 GPU",
+            "parallelism": parallelism_note(gpus),
             **({"algorithm": args.algorithm, "local_optimizer": args.optimizer,
                 "lost_prob": args.lost_prob, "mu": args.objective} if args is not None else {})}
 
@@ -475,7 +506,7 @@ def roofline_of(args, w, run, models_ms) -> dict:
 def run_native(args, w, rank: int, world: int):
     import torch
 
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    local = local_device(int(os.environ.get("LOCAL_RANK", "0")), torch.cuda.device_count())
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
@@ -516,7 +547,7 @@ def run_native(args, w, rank: int, world: int):
             "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": workload_config(w, world, args, dev), "roofline": roofline, "cpu_baseline": cpu,
-            "e2e": e2e, "gpu_launches": 2 * T * args.steps, "clocks": clocks,
+            "e2e": e2e, "gpu_launches": world * 2 * T * args.steps, "clocks": clocks,
             "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1),
             "fused_steps": fused, "per_workload": per_workload}
     print(json.dumps(line), flush=True)
@@ -553,7 +584,7 @@ def run_per_workload(args, head, dev, stream, rank: int, world: int, local: int)
                         "n_workers": w.n, "tree": cfg["tree"], "d": w.d, "steps": args.steps,
                         "warmup": args.warmup, "l2": cfg["l2"],
                         "roofline": roofline_of(args, w, run, models_ms), "clocks": clocks,
-                        "gpu_launches": 2 * len(run.trees) * args.steps})
+                        "gpu_launches": world * 2 * len(run.trees) * args.steps})
         del run, one_step
         gc.collect()
         torch.cuda.empty_cache()
@@ -643,7 +674,7 @@ def run_graphed(args, w, run, dev, stream, rank: int, world: int):
                          "peak": peak, "unit": "GB/s",
                          "frac": round(alg / (per_step / 1e3) / 1e9 / peak, 4), "traffic": None,
                          "kernel": "whole step (graph replay)"},
-            "cpu_baseline": None, "e2e": None, "gpu_launches": 2 * len(run.trees) * args.steps,
+            "cpu_baseline": None, "e2e": None, "gpu_launches": world * 2 * len(run.trees) * args.steps,
             "clocks": clocks.summary()}
     print(json.dumps(line), flush=True)
 
@@ -844,8 +875,10 @@ def main(argv=None):
     if world > 1:
         import torch
         import torch.distributed as dist
-        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
-        dist.init_process_group("nccl")
+        n_dev = torch.cuda.device_count()
+        torch.cuda.set_device(local_device(int(os.environ.get("LOCAL_RANK", "0")), n_dev))
+        local_world = int(os.environ.get("LOCAL_WORLD_SIZE", str(world)))
+        dist.init_process_group(process_group_backend(local_world, n_dev))
     try:
         run_native(args, w, rank, world)
     finally:

@@ -73,3 +73,17 @@ def test_shard_offsets_are_quad_aligned():
             c0 = bench.shard_offset(r, d)
             assert c0 % 4 == 0 and c0 >= r * d
             assert bench.shard_offset(r + 1, d) - c0 >= d
+
+
+def test_rank_placement_and_backend():
+    """One GPU per local rank: rank i on GPU i over NCCL; more ranks than
+    GPUs: round robin over them, host collectives over gloo."""
+    import bench
+    assert [bench.local_device(r, 8) for r in range(8)] == list(range(8))
+    assert [bench.local_device(r, 1) for r in range(4)] == [0, 0, 0, 0]
+    assert [bench.local_device(r, 2) for r in range(4)] == [0, 1, 0, 1]
+    assert bench.process_group_backend(8, 8) == "nccl"
+    assert bench.process_group_backend(1, 1) == "nccl"
+    assert bench.process_group_backend(2, 1) == "gloo"
+    with pytest.raises(RuntimeError):
+        bench.local_device(0, 0)
