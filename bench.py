@@ -11,15 +11,18 @@ per-step working set (82.7 GB moved) is far larger than L2, so no flush is
 needed between steps.  Inputs are seeded synthetic quadratics.
 
 Prints one JSON line.  `value` is whole-job steps/s with the state resident
-in HBM; `e2e` is the same metric through relay_step with the state in pinned
-host buffers (copies inside the timed region); `roofline` is the fused
+in HBM; `e2e` is the same metric through relay_step_host with the state in
+pinned host buffers (copies inside the timed region); `roofline` is the step
 kernel's algorithmic HBM bytes per launch over its CUDA-event duration;
 `cpu_baseline` times the plain CPU oracle on a bounded coordinate sample,
-on every host core (one slice per thread) and on one thread.
+on every host core (one slice per thread) and on one thread; `metrics` is the
+consensus distance and the average model's distance to the optimum after the
+timed steps, over every rank's slice.
 
 Multi-GPU (torchrun, one rank per GPU): every rank runs the same workload on
 its own d-slice of one longer model vector (coordinates are independent, so
-there is no data-path collective; weak scaling).  With more local ranks than
+there is no data-path collective; weak scaling; the one collective, after the
+timed region, sums the ranks' metrics).  With more local ranks than
 visible GPUs the ranks share them round robin and the process group uses
 gloo (a functional check of the multi-rank path; such a line is no scaling
 figure).  `--impl reference` times the CPU oracle instead (rank 0 only).
@@ -83,6 +86,41 @@ def process_group_backend(local_world: int, n_devices: int) -> str:
     collectives) where ranks share one, which NCCL refuses.  The path has no
     data-path collective, only the barrier and the max over ranks."""
     return "nccl" if local_world <= n_devices else "gloo"
+
+
+def combine_slice_metrics(parts) -> tuple:
+    """Whole-vector (consensus distance, distance of the average model to the
+    optimum) from the metrics of coordinate slices.  relay_metrics gives each
+    as a mean over its slice's coordinates (1/(n d) sum_i ||x_i - xbar||^2 and
+    ||xbar - mubar||^2 / d), so the whole vector's is the mean of the slices'
+    weighted by their widths.  parts: [(d_slice, consensus, distance)]."""
+    total = sum(p[0] for p in parts)
+    if total <= 0:
+        return 0.0, 0.0
+    return (sum(p[0] * p[1] for p in parts) / total, sum(p[0] * p[2] for p in parts) / total)
+
+
+def sharded_metrics(run, world: int) -> dict:
+    """The run's metrics over every rank's slice (and tree window): the one
+    collective of the d-sharded path, an all-reduce of three doubles, taken
+    after the timed region."""
+    import torch
+    m = run.metrics().cpu().tolist()
+    # width-weighted sums over this rank's tree windows, then over the ranks
+    sums = [sum(tr.d * m[k][0] for k, tr in enumerate(run.trees)),
+            sum(tr.d * m[k][1] for k, tr in enumerate(run.trees)),
+            float(sum(tr.d for tr in run.trees))]
+    if world > 1:
+        import torch.distributed as dist
+        dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+        t = torch.tensor(sums, dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        sums = t.cpu().tolist()
+    c, dist_opt = combine_slice_metrics([(sums[2], sums[0] / sums[2], sums[1] / sums[2])] if sums[2] > 0 else [])
+    return {"consensus_distance": c, "distance_to_optimum": dist_opt, "after_steps": run.t,
+            "coordinates": int(sums[2]),
+            "note": "relay_metrics per rank and tree window, combined by slice width"
+                    + (" with one all-reduce of 3 doubles after the timed region" if world > 1 else "")}
 
 
 def barrier(world: int):
@@ -522,6 +560,7 @@ def run_native(args, w, rank: int, world: int):
     steps_per_s = world * args.steps / (total_ms / 1e3)
     roofline = roofline_of(args, w, run, models_ms) if rank == 0 else None
     alg_bytes = w.bytes_per_step()
+    metrics = sharded_metrics(run, world)
 
     # several steps per call, on the resident run (before run_e2e frees it)
     fused = run_fused(args, w, run, dev, stream, world) if args.fused_steps > 0 else None
@@ -549,7 +588,7 @@ def run_native(args, w, rank: int, world: int):
             "config": workload_config(w, world, args, dev), "roofline": roofline, "cpu_baseline": cpu,
             "e2e": e2e, "gpu_launches": world * 2 * T * args.steps, "clocks": clocks,
             "hbm_gbs_step": round(alg_bytes * world * args.steps / (total_ms / 1e3) / 1e9, 1),
-            "fused_steps": fused, "per_workload": per_workload}
+            "fused_steps": fused, "per_workload": per_workload, "metrics": metrics}
     print(json.dumps(line), flush=True)
 
 

@@ -48,3 +48,7 @@ def test_native_arm_two_ranks_on_one_gpu():
     assert abs(line["value"] - 2 * 3 / (line["ms_per_step"] * 3 / 1e3)) <= 1e-3 * line["value"]
     r = line["roofline"]
     assert r["bound"] == "hbm" and r["achieved"] > 0 and r["kernel"] == "relay_models_kernel"
+    # the metrics of both ranks' slices, combined by the one all-reduce
+    m = line["metrics"]
+    assert m["coordinates"] == 2 * 9_231_114 and m["after_steps"] == 3 + 3
+    assert 0 < m["consensus_distance"] < 10 and 0 < m["distance_to_optimum"] < 10

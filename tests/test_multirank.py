@@ -87,3 +87,64 @@ def test_rank_placement_and_backend():
     assert bench.process_group_backend(2, 1) == "gloo"
     with pytest.raises(RuntimeError):
         bench.local_device(0, 0)
+
+
+def _oracle_metrics(x: np.ndarray, mu: np.ndarray):
+    """Consensus distance 1/(n d) sum_i ||x_i - xbar||^2 and ||xbar - mubar||^2 / d
+    of fp64 models x [n][d] and centres mu [n][d], straight from the definition."""
+    xbar = x.mean(axis=0)
+    mubar = mu.mean(axis=0)
+    return float(((x - xbar) ** 2).sum(axis=0).mean() / x.shape[0]), float(((xbar - mubar) ** 2).mean())
+
+
+def test_slice_metrics_combine_to_the_whole_vector():
+    """Per-slice metrics weighted by slice width equal the whole vector's."""
+    import bench
+    from oracle import oracle
+    from paper_2110_04175_gb300 import workloads as wl
+    w = wl.Workload("bin9", 9, wl.binary_tree(9), 1000, wl.identity_mix(9), 1.0, 0.1, 0.1, 0.1, 7)
+    st = oracle.State(w.n, w.edges, 3 * w.d)
+    st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
+    st.advance(w.steps, w.lr, w.sigma, w.seed, w.mode)
+    whole = _oracle_metrics(st.x, st.mu)
+    cuts = [0, 400, 1004, 3000]  # ragged slices
+    parts = [(b - a, *_oracle_metrics(st.x[:, a:b], st.mu[:, a:b])) for a, b in zip(cuts, cuts[1:])]
+    got = bench.combine_slice_metrics(parts)
+    assert np.allclose(got, whole, rtol=1e-12, atol=0)
+    assert whole[0] > 0 and whole[1] > 0
+
+
+class _SliceRun:
+    """Stands in for a RelayRun in bench.sharded_metrics: the metrics of its
+    tree windows and their widths."""
+
+    def __init__(self, windows, t):
+        self.trees = [type("W", (), {"d": d})() for d, _, _ in windows]
+        self._m = torch.tensor([[c, m] for _, c, m in windows], dtype=torch.float64)
+        self.t = t
+
+    def metrics(self):
+        return self._m
+
+
+def _metrics_worker(rank, world, port, result_dir):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        import bench
+        windows = [[(300, 0.5, 2.0), (700, 1.5, 1.0)], [(1000, 3.0, 4.0)]][rank]
+        got = bench.sharded_metrics(_SliceRun(windows, 12), world)
+        want = bench.combine_slice_metrics([(300, 0.5, 2.0), (700, 1.5, 1.0), (1000, 3.0, 4.0)])
+        assert got["coordinates"] == 2000 and got["after_steps"] == 12
+        assert np.allclose([got["consensus_distance"], got["distance_to_optimum"]], want, rtol=1e-15)
+        if rank == 0:
+            open(os.path.join(result_dir, "ok"), "w").write("ok")
+    finally:
+        dist.destroy_process_group()
+
+
+def test_sharded_metrics_all_reduce_two_ranks(tmp_path):
+    port = _free_port()
+    mp.spawn(_metrics_worker, args=(2, port, str(tmp_path)), nprocs=2, join=True)
+    assert (tmp_path / "ok").exists()
