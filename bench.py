@@ -419,10 +419,10 @@ def make_run(args, w, dev, c0: int):
 
 
 def make_stepper(args, w, run, stream, rank: int):
-    """one_step(ev): one step of `run` on `stream`; ev (per tree window: three
-    CUDA events) brackets the counter kernel and the step kernel.  Several
-    tree windows (double binary trees) are one relay_step_windows call (one
-    counter launch, one step-kernel launch), timed as a whole."""
+    """one_step(ev): one step of `run` on `stream` through the library's step
+    call -- relay_step (the step kernel a programmatic dependent of the
+    counter kernel), or relay_step_windows for several tree windows --
+    bracketed by the CUDA events ev = (start, end) when given."""
     import numpy as np
     import torch
 
@@ -435,27 +435,11 @@ def make_stepper(args, w, run, stream, rank: int):
         for tr in run.trees:
             if args.lost_prob > 0:  # messages lost in transit this step (Section 4.4)
                 rs.relay_set_lost_messages(tr.h, lost_rng.random(tr.E) < args.lost_prob)
-        if len(run.trees) > 1:
-            if ev is not None:
-                ev[0][0].record(stream)
-                ev[0][1].record(stream)
-            run.step(w.lr, w.seed, stream)
-            if ev is not None:
-                ev[-1][2].record(stream)
-            torch.cuda.nvtx.range_pop()
-            return
-        tr = run.trees[0]
         if ev is not None:
-            ev[0][0].record(stream)
-        rs.relay_step_counts(tr.h, tr.counts, stream)
+            ev[0].record(stream)
+        run.step(w.lr, w.seed, stream)
         if ev is not None:
-            ev[0][1].record(stream)
-        rs.relay_step_models(tr.h, run._x(tr), tr.msg[tr.cur], tr.msg[1 - tr.cur], tr.counts,
-                             w.lr, w.seed, run.t, stream)
-        if ev is not None:
-            ev[0][2].record(stream)
-        tr.cur = 1 - tr.cur
-        run.t += 1
+            ev[1].record(stream)
         torch.cuda.nvtx.range_pop()
 
     return one_step
@@ -463,16 +447,17 @@ def make_stepper(args, w, run, stream, rank: int):
 
 def time_steps(args, w, run, one_step, dev, stream, rank: int, world: int, local: int):
     """Times args.steps steps (after the warm-up already run): (total ms,
-    max over ranks; step-kernel ms of every step; clock summary)."""
+    max over ranks; the duration of every step; clock summary).  Each step
+    is one library call bracketed by two CUDA events on the launching
+    stream; its duration is the step kernel's plus whatever of the counter
+    kernel the programmatic dependent launch does not overlap."""
     import torch
-    T = len(run.trees)
     # a working set that fits in L2 is evicted before every timed step (a
     # memset of twice the L2), and the steps are then timed one by one
     flush = None
     if l2_flush_needed(w, args, dev):
         flush = torch.empty(2 * l2_bytes(dev), dtype=torch.uint8, device=dev)
-    events = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(T)]
-              for _ in range(args.steps)]
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
     torch.cuda.synchronize(dev)
     barrier(world)
     torch.cuda.synchronize(dev)
@@ -484,17 +469,13 @@ def time_steps(args, w, run, one_step, dev, stream, rank: int, world: int, local
         torch.cuda.synchronize(dev)
     barrier(world)
     torch.cuda.synchronize(dev)
+    step_ms = [events[k][0].elapsed_time(events[k][1]) for k in range(args.steps)]
     if flush is None:
-        total_ms = events[0][0][0].elapsed_time(events[-1][-1][2])
+        total_ms = events[0][0].elapsed_time(events[-1][1])
     else:
-        total_ms = sum(events[k][0][0].elapsed_time(events[k][-1][2]) for k in range(args.steps))
+        total_ms = sum(step_ms)
         del flush
-    # step-kernel time per step (several windows: the whole step)
-    if T == 1:
-        models_ms = [events[k][0][1].elapsed_time(events[k][0][2]) for k in range(args.steps)]
-    else:
-        models_ms = [events[k][0][1].elapsed_time(events[k][-1][2]) for k in range(args.steps)]
-    return reduce_max(total_ms, world), models_ms, clocks.summary()
+    return reduce_max(total_ms, world), step_ms, clocks.summary()
 
 
 def kernel_name_of(run) -> str:
@@ -502,12 +483,15 @@ def kernel_name_of(run) -> str:
     name = ("relay_nodes_kernel" if rs.relay_get_kernel(run.h) == rs.RELAY_KERNEL_NODES
             else "relay_models_kernel")
     T = len(run.trees)
-    return name if T == 1 else f"{name} over {T} tree windows in one launch (relay_step_windows; whole step timed)"
+    return name if T == 1 else f"{name} over {T} tree windows in one launch (relay_step_windows)"
 
 
 def roofline_of(args, w, run, models_ms) -> dict:
-    """The step kernel's algorithmic HBM bytes per launch over its mean
-    CUDA-event time, against the measured copy bandwidth."""
+    """The step kernel's algorithmic HBM bytes per launch over the mean
+    CUDA-event time of the step call that launches it (the step kernel plus
+    the part of the one-CTA counter kernel its programmatic dependent launch
+    does not overlap: an upper bound on the kernel's own time), against the
+    measured copy bandwidth."""
     peaks = measured_peaks()
     peak = peaks.get("hbm_gbs")
     peak_src = "measured" if peak else "fallback"
@@ -532,6 +516,8 @@ def roofline_of(args, w, run, models_ms) -> dict:
                 "achieved_design_bytes": round(moved / (mean_models_ms / 1e3) / 1e9, 1),
                 "launch_ms_mean": round(mean_models_ms, 4),
                 "launch_ms_min": round(min(models_ms), 4),
+                "timed": "each relay_step call between two CUDA events on its stream (counter kernel, then "
+                         "the step kernel as its programmatic dependent)",
                 "nominal_peak": NOMINAL_HBM_GBS,
                 "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4)}
     if roofline["traffic"]:
