@@ -10,7 +10,7 @@ them when RELAY_PARITY_LOG names a file.
 The fp32 path differs from the fp64 definition only by rounding: a float32
 restatement of the step stays within 1e-6 of the oracle on every workload
 (10x below the bar), so 1e-5 leaves room for the GPU's own summation order
-and its fp32 logf/sincospif in the noise.
+and its fp32 normals (within NORMAL_ABS_ERR of the oracle's).
 """
 from __future__ import annotations
 
@@ -23,6 +23,19 @@ import paper_2110_04175_gb300 as rs
 from oracle import oracle
 
 RTOL = 1e-5
+
+# How far a normal drawn on the GPU can sit from the oracle's fp64 Box-Muller
+# of the same Philox uniforms.  The GPU forms z = r (cos, sin)(theta) with
+# r = sqrt(-2 ln u), u >= 2^-24 (so r <= sqrt(48 ln 2) = 5.77), using CUDA's
+# logf, sqrt.approx and the fast __sincosf on theta = 2 pi u - pi, computed
+# with one fp32 fma.  Terms, at r = 5.77:
+#   theta's error: |pi_f - pi| + half an ulp at |theta| <= pi, 3.3e-7, times r     1.9e-6
+#   __sincosf: at most 2^-21.41 absolute on [-pi, pi] (CUDA's stated bound), times r 2.1e-6
+#   r: logf (1 ulp) and sqrt.approx (taken as 2^-22 relative), times |z|            1.6e-6
+#   the product's rounding, 2^-24 |z|                                               0.4e-6
+# test_normal_generator_error_within_derived_bound measures it on 8.4M normals
+# (largest deviation 1.6e-6).
+NORMAL_ABS_ERR = 6e-6
 
 # When set, the full-size parity tests append one JSON line per compared
 # array to this file: the metric above and the plain errors beside it.
@@ -72,6 +85,14 @@ def parity_report(g: np.ndarray, r: np.ndarray) -> dict:
     out["rel_max_big"] = float(np.max(diff[big] / a[big])) if big.any() else None
     out["floor_share"] = float(np.mean(a < rms))
     return out
+
+
+def generated_input_error(mix, mu_scale: float, sigma: float, x0_std: float) -> np.ndarray:
+    """Per worker ([n][1]), how far the gradient's generated inputs may sit
+    from the oracle's: mu_i = mu_scale sum_k mix_ik N_k, sigma xi_i and the
+    shared x^0 = x0_std N are normals, each within NORMAL_ABS_ERR."""
+    mix = np.abs(np.asarray(mix, dtype=np.float64))
+    return ((mu_scale * mix.sum(axis=1) + sigma + x0_std) * NORMAL_ABS_ERR)[:, None]
 
 
 def record_parity(label: str, array: str, g, r):
@@ -180,7 +201,7 @@ def compare_ranges(run: rs.RelayRun, w, ranges, steps: int, mode: int | None = N
 
 
 def adam_step_bound(x, mu, xi, sigma: float, m, v, lr: float, beta1: float, beta2: float, eps: float,
-                    t: int) -> np.ndarray:
+                    t: int, dnoise=0.0) -> np.ndarray:
     """Per coordinate, how far fp32 rounding can move one Adam step (t from
     0) of any worker, from the oracle's state before the step (x, mu, the
     noise xi) and after it (first and second moments m, v), all [n][len].
@@ -193,11 +214,15 @@ def adam_step_bound(x, mu, xi, sigma: float, m, v, lr: float, beta1: float, beta
     -lr g / (|g| + eps), in effect -lr sign(g) when eps is tiny: within
     rounding of zero the sign is a decision that two precisions may take
     differently, a difference of 2 lr.  dg is the fp32 rounding of the
-    gradient's terms, 2^-23 (|x| + |mu| + sigma |xi|).  The relay and
-    rebuild only average, so the largest worker's value bounds the step's
-    effect on every worker; summed over steps it bounds the trajectory."""
+    gradient's terms, 2^-23 (|x| + |mu| + sigma |xi|), plus `dnoise`, how far
+    the generated inputs of the gradient (the centres, the noise and the
+    initial model, drawn as normals) may sit from the oracle's:
+    (mu_scale sum_k |mix_ik| + sigma + x0_std) NORMAL_ABS_ERR per worker
+    ([n][1], or a scalar).  The relay and rebuild only average, so the
+    largest worker's value bounds the step's effect on every worker; summed
+    over steps it bounds the trajectory."""
     g = (x - mu) + sigma * xi
-    dg = 2.0 ** -23 * (np.abs(x) + np.abs(mu) + sigma * np.abs(xi))
+    dg = 2.0 ** -23 * (np.abs(x) + np.abs(mu) + sigma * np.abs(xi)) + dnoise
     k = t + 1
     denom = np.sqrt(v / (1.0 - beta2 ** k)) + eps
     du = lr * (1.0 - beta1) / (1.0 - beta1 ** k) * dg / denom

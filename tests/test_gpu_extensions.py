@@ -11,7 +11,8 @@ import paper_2110_04175_gb300 as rs
 from oracle import oracle
 from paper_2110_04175_gb300 import build as rs_build
 from paper_2110_04175_gb300 import workloads as wl
-from tests.gpu_util import RTOL, adam_step_bound, c8_sample, parallel_map, parity_error, record_parity
+from tests.gpu_util import (RTOL, adam_step_bound, c8_sample, generated_input_error, parallel_map, parity_error,
+                            record_parity)
 
 pytestmark = pytest.mark.gpu
 
@@ -109,11 +110,12 @@ def adam_rounding_bound(w, start, length, steps, beta1, beta2, eps):
     st.init(w.x0_std, w.seed, w.mix.astype(np.float64), w.mu_scale, w.mu_seed)
     mu = st.mu.copy()
     bound = np.zeros(length)
+    dnoise = generated_input_error(w.mix, w.mu_scale, sigma, w.x0_std)
     for t in range(steps):
         x = st.x.copy()
         xi = np.stack([oracle.normals(w.seed, start, length, row=i, step=t, stream=0) for i in range(w.n)])
         st.advance(1, lr, sigma, w.seed, w.mode, opt=oracle.OPT_ADAM, beta1=beta1, beta2=beta2, eps=eps)
-        bound += adam_step_bound(x, mu, xi, sigma, st.s1, st.s2, lr, beta1, beta2, eps, t)
+        bound += adam_step_bound(x, mu, xi, sigma, st.s1, st.s2, lr, beta1, beta2, eps, t, dnoise)
     return st, bound
 
 

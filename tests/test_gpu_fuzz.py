@@ -8,7 +8,8 @@ nodes' received sums, then compares every coordinate of the models
 and messages, the counters (bit-exact) and the mean-estimation counts with
 the oracle.  Adam cases hold every element to the 1e-5 bar plus the fp32
 rounding bound derived from Adam's arithmetic (gpu_util.adam_step_bound,
-summed over the steps; n times that for messages): Adam's update is about lr
+with the generated inputs' error gpu_util.generated_input_error, summed over
+the steps; n times that for messages): Adam's update is about lr
 whatever the gradient, so its own rounding accumulates with lr, the steps and,
 in messages, the workers summed.  They draw eps = 1e-2, which keeps the first
 step from being a sign decision (that case is the full-size Adam test's).
@@ -23,7 +24,7 @@ import paper_2110_04175_gb300 as rs
 from oracle import oracle
 from paper_2110_04175_gb300 import build as rs_build
 from paper_2110_04175_gb300 import workloads as wl
-from tests.gpu_util import RTOL, adam_step_bound, parity_error
+from tests.gpu_util import RTOL, adam_step_bound, generated_input_error, parity_error
 
 pytestmark = pytest.mark.gpu
 
@@ -53,7 +54,7 @@ def draw(case: int) -> dict:
         mix = rng.random((n, int(rng.integers(1, 9)))).astype(np.float32)
     opt = rng.choice(["sgd", "nesterov", "adam"], p=[.5, .25, .25])
     algo = rng.choice(["relaysgd", "grad", "dme"], p=[.6, .2, .2])
-    return dict(n=n, shape=str(shape), edges=np.asarray(edges, np.int32).reshape(-1, 2),
+    c = dict(n=n, shape=str(shape), edges=np.asarray(edges, np.int32).reshape(-1, 2),
                 d=int(rng.integers(1, 3000)), c0=4 * int(rng.integers(0, 50_000)), mode=int(rng.integers(0, 2)),
                 objective=str(rng.choice(["stored", "generated"])), mix=mix, mixkind=str(mixkind),
                 opt=str(opt), beta1=float(rng.uniform(0.5, 0.95)), beta2=float(rng.uniform(0.9, 0.999)),
@@ -64,6 +65,10 @@ def draw(case: int) -> dict:
                 seed=int(rng.integers(0, 2**40)), mu_seed=int(rng.integers(0, 2**40)),
                 # drawn from streams of their own, so the other draws of each case are unchanged
                 received_sums=bool(np.random.default_rng(5000 + case).integers(0, 2)))
+    # regenerated centres take at most 1024 mixture non-zeros (relay_set_objective_generated)
+    if c["objective"] == "generated" and np.count_nonzero(c["mix"]) > 1024:
+        c["objective"] = "stored"
+    return c
 
 
 @pytest.mark.parametrize("case", range(120))
@@ -92,6 +97,7 @@ def test_random_configuration_against_oracle(case):
     lr, sigma = float(np.float32(c["lr"])), float(np.float32(c["sigma"]))
     adam = c["opt"] == "adam"
     bound = np.zeros(d)
+    dnoise = generated_input_error(c["mix"], c["mu_scale"], sigma, c["x0_std"])
     for t in range(c["steps"]):
         lost = (rng.random(E) < c["lost_p"]).astype(np.uint8)
         if c["lost_p"] > 0:
@@ -102,7 +108,8 @@ def test_random_configuration_against_oracle(case):
                    algo=algo, **kw)
         if adam:
             xi = np.stack([oracle.normals(c["seed"], c["c0"], d, row=i, step=t, stream=0) for i in range(n)])
-            bound += adam_step_bound(x, st.mu, xi, sigma, st.s1, st.s2, lr, c["beta1"], c["beta2"], 1e-2, t)
+            bound += adam_step_bound(x, st.mu, xi, sigma, st.s1, st.s2, lr, c["beta1"], c["beta2"], 1e-2, t,
+                                     dnoise)
     torch.cuda.synchronize()
     info = {k: v for k, v in c.items() if k not in ("edges", "mix")}
 
