@@ -995,11 +995,35 @@ __global__ void relay_fill_mu_kernel(float* mu, const float* mix, int n, int K, 
 // paper's analysis, Section 4): per coordinate c, with xbar = mean_i x_i and
 // mubar = mean_i mu_i,
 //   xi   += sum_i (x_i - xbar)^2        dist += (xbar - mubar)^2
-// accumulated in double.  Pass 1: each block reduces its share of the
-// coordinates (grid-stride, fixed order) into partials[2 blockIdx];
-// pass 2 sums the partials in a fixed order, so the result is deterministic.
+// Pass 1: each block reduces its share of the coordinates (grid-stride,
+// fixed order) into partials[2 blockIdx]; pass 2 sums the partials in a
+// fixed order, so the result is deterministic.  Within a coordinate the
+// sums over the workers run in fp32 pairs (below) and only the coordinate's
+// totals in double: the GB300's fp64 rate is a small fraction of its fp32
+// rate, and per-worker fp64 arithmetic made the metrics fp64-bound.
 constexpr int kMetricsThreads = 256;
 constexpr int kMetricsMaxBlocks = 1024;
+
+// A running fp32 sum kept as the unevaluated pair s + c (Neumaier's
+// compensated summation): c gathers every addition's exact rounding error,
+// so the pair carries about twice fp32's precision.  The _rn intrinsics
+// keep the compiler from contracting or reordering the error terms.
+struct PairSum {
+    float s = 0.0f, c = 0.0f;
+    __device__ __forceinline__ void add(float v) {
+        const float t = __fadd_rn(s, v);
+        const float e = (fabsf(s) >= fabsf(v)) ? __fadd_rn(__fsub_rn(s, t), v) : __fadd_rn(__fsub_rn(v, t), s);
+        c = __fadd_rn(c, e);
+        s = t;
+    }
+    __device__ __forceinline__ double value() const { return static_cast<double>(s) + static_cast<double>(c); }
+};
+
+// The exact rounding error of a + b, given s = fl(a + b) (Knuth's TwoSum).
+__device__ __forceinline__ float sum_error(float a, float b, float s) {
+    const float bb = __fsub_rn(s, a);
+    return __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
 
 __device__ __forceinline__ double block_sum(double v, double* red) {
     for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
@@ -1020,25 +1044,43 @@ relay_metrics_kernel(const __grid_constant__ Objective obj, const __grid_constan
     __shared__ double red[kMetricsThreads / 32];
     double xi = 0.0, dist = 0.0;
     const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    const double inv_n = 1.0 / n;
     for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < a.nquads; q += stride) {
-        double xs[4] = {0, 0, 0, 0}, ms[4] = {0, 0, 0, 0};
+        PairSum xs[4], ms[4];
         for (int i = 0; i < n; ++i) {
             const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
             const float4 mv = centre<OBJ>(obj, mu_key, a, i, q, nullptr, 0);
-            xs[0] += xv.x; xs[1] += xv.y; xs[2] += xv.z; xs[3] += xv.w;
-            ms[0] += mv.x; ms[1] += mv.y; ms[2] += mv.z; ms[3] += mv.w;
+            xs[0].add(xv.x); xs[1].add(xv.y); xs[2].add(xv.z); xs[3].add(xv.w);
+            ms[0].add(mv.x); ms[1].add(mv.y); ms[2].add(mv.z); ms[3].add(mv.w);
         }
-        double xb[4], ss[4] = {0, 0, 0, 0};
-        for (int k = 0; k < 4; ++k) xb[k] = xs[k] / n;
+        // xbar as the fp32 pair hi + lo
+        float hi[4], lo[4];
+        double xb[4];
+        for (int k = 0; k < 4; ++k) {
+            xb[k] = xs[k].value() * inv_n;
+            hi[k] = static_cast<float>(xb[k]);
+            lo[k] = static_cast<float>(xb[k] - static_cast<double>(hi[k]));
+        }
+        // sum_i (x_i - xbar)^2: x_i - hi exactly as t + its rounding error,
+        // less lo; t^2 exactly as p + its fma remainder
+        PairSum sq[4];
+        float sq_lo[4] = {0.f, 0.f, 0.f, 0.f};
         for (int i = 0; i < n; ++i) {
             const float4 xv = *reinterpret_cast<const float4*>(a.x + i * a.ld_x + 4 * q);
-            const double dv[4] = {xv.x - xb[0], xv.y - xb[1], xv.z - xb[2], xv.w - xb[3]};
-            for (int k = 0; k < 4; ++k) ss[k] += dv[k] * dv[k];
+            const float xk[4] = {xv.x, xv.y, xv.z, xv.w};
+            for (int k = 0; k < 4; ++k) {
+                const float t = __fsub_rn(xk[k], hi[k]);
+                const float dl = __fsub_rn(sum_error(xk[k], -hi[k], t), lo[k]);
+                const float p = __fmul_rn(t, t);
+                const float pe = __fmaf_rn(t, t, -p);
+                sq[k].add(p);
+                sq_lo[k] = __fadd_rn(sq_lo[k], __fmaf_rn(__fmul_rn(2.0f, t), dl, pe));
+            }
         }
         for (int k = 0; k < 4; ++k)
             if (4 * q + k < d) {
-                xi += ss[k];
-                const double e = xb[k] - ms[k] / n;
+                xi += sq[k].value() + static_cast<double>(sq_lo[k]);
+                const double e = xb[k] - ms[k].value() * inv_n;
                 dist += e * e;
             }
     }
