@@ -159,16 +159,17 @@ def test_small_cases_every_coordinate(shape, n, d, mode, objective, kernel):
     assert ex <= RTOL and em <= RTOL, (ex, em)
 
 
+@pytest.mark.parametrize("kernel", ["walk", "nodes"])
 @pytest.mark.parametrize("mix", ["identity", "dirichlet", "dense"])
-def test_generated_objective_bit_identical_to_stored(mix):
-    """Regenerating mu in the fused kernel (per-row normals or cached centres)
-    gives exactly the bits of the stored, pre-filled mu."""
+def test_generated_objective_bit_identical_to_stored(mix, kernel):
+    """Regenerating mu in the step kernel (per-row normals or cached centres)
+    gives exactly the bits of the stored, pre-filled mu, on both step kernels."""
     n, d = 16, 20_000
     m = {"identity": wl.identity_mix(n), "dirichlet": wl.dirichlet_mix(n, 10, 0.1, seed=3),
          "dense": np.random.default_rng(0).random((n, 24)).astype(np.float32)}[mix]
     w = wl.Workload("mix", n, wl.random_tree(n, 2), d, m, 1.3, 0.05, 0.05, 0.1, 15)
-    a = gpu_run(w, w.steps, objective="stored")
-    b = gpu_run(w, w.steps, objective="generated")
+    a = gpu_run(w, w.steps, objective="stored", kernel=kernel)
+    b = gpu_run(w, w.steps, objective="generated", kernel=kernel)
     assert torch.equal(a.x, b.x) and torch.equal(a.messages, b.messages)
 
 
