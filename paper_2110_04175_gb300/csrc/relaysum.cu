@@ -603,8 +603,16 @@ __device__ __forceinline__ void walk(const Program& prog, const ModelArgs& a, co
 // each copy reads its window's program and arguments at fixed parameter
 // offsets (constant operands), as the one-window kernel does; the grid's
 // first `split` CTAs take window 0.
+// Resident CTAs of 128 threads per SM the walk's registers are budgeted for
+// (0: no bound, the compiler's choice, 72 registers and 7 CTAs for the
+// stored-centre walk).  The wide-node variant runs 8 CTAs with 64 registers:
+// 6.17 -> 6.08 ms per step on the 64-worker star, while the same budget
+// slowed every narrow tree (double16 +11 %, binary32 +4 %; same-box A/B).
+template <bool WIDE>
+constexpr int kWalkMinCtas = WIDE ? 8 : 0;
+
 template <int OBJ, int OPT, int NT, bool WIDE>
-__global__ void __launch_bounds__(128)
+__global__ void __launch_bounds__(128, kWalkMinCtas<WIDE>)
 relay_models_kernel(const __grid_constant__ Windows<NT> win, const __grid_constant__ Objective obj,
                     const __grid_constant__ PhiloxKey mu_key) {
     extern __shared__ float4 slot_mem[];
