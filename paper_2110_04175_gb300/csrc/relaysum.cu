@@ -725,10 +725,11 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
         xn = *reinterpret_cast<const float4*>(xrow + 4 * q);
         if (OBJ == relaysum::kMuStored) mn = ld_stream(murow + 4 * q);
     }
-    // x and mu are not written by the counter kernel; the counters are
-    wait_for_prior_grid();
-    rebuild_factors(prog, a, s_scale, s_fill);
-    __syncthreads();
+    // Phase 1 needs no counter: the first block's runs before the wait for the
+    // counter kernel (programmatic dependent launch), overlapping it; only the
+    // rebuild factors of phase 2 need the counters, which the counter kernel
+    // writes (it writes nothing phase 1 reads).
+    bool counted = false;
     int parity = 0;
     for (int64_t b = blockIdx.x; b < nblk; b += gridDim.x, q += qstep, parity ^= 1) {
         float4* const m_new = parity ? buf1 : buf0;
@@ -738,14 +739,12 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
             xn = *reinterpret_cast<const float4*>(xrow + 4 * (q + qstep));
             if (OBJ == relaysum::kMuStored) mn = ld_stream(murow + 4 * (q + qstep));
         }
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 xh = make_float4(0.f, 0.f, 0.f, 0.f);
         if (active) {
             const float4 mv = (OBJ == relaysum::kMuStored) ? ms : centre<kObj>(obj, mu_key, a, i, q, nullptr, 0);
             const float4 z = normal4(a.q0 + static_cast<uint32_t>(q), static_cast<uint32_t>(i), a.step, 0u,
                                      a.key);
-            const float4 xh = relayed_value<OPT>(a, i, q, xv, mv, z);
-            acc = xh;
-            if (s_fill[i] != 0.0f) acc = add4(scale4(xv, s_fill[i]), xh);
+            xh = relayed_value<OPT>(a, i, q, xv, mv, z);
             switch (r.deg) {
                 case 0: break;
                 case 1: node_small<1>(prog, r, a, q, xh, m_new, qb); break;
@@ -755,8 +754,16 @@ relay_nodes_kernel(const __grid_constant__ Program prog, const __grid_constant__
                 default: node_wide(prog, r, a, i, q, xh, m_new, m_old, qb); break;
             }
         }
-        __syncthreads();
+        if (!counted) {
+            wait_for_prior_grid();
+            rebuild_factors(prog, a, s_scale, s_fill);
+            counted = true;
+        }
+        __syncthreads();  // also publishes the factors
         if (active) {
+            // the rebuild sum starts from fill_i x_i + x^{t+1/2}, as in the walk
+            float4 acc = xh;
+            if (s_fill[i] != 0.0f) acc = add4(scale4(xv, s_fill[i]), xh);
             if (a.rsum && r.deg > kRegDeg) {  // and the wide node's received sum S_i^t, in the same order
                 float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
                 for (int k = 0; k < r.deg; ++k) {
