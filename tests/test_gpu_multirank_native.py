@@ -52,3 +52,32 @@ def test_native_arm_two_ranks_on_one_gpu():
     m = line["metrics"]
     assert m["coordinates"] == 2 * 9_231_114 and m["after_steps"] == 3 + 3
     assert 0 < m["consensus_distance"] < 10 and 0 < m["distance_to_optimum"] < 10
+
+
+@pytest.mark.gpu
+def test_native_arm_two_ranks_with_every_leg():
+    """The legs the default command adds to the headline -- the per-workload
+    lines, the several-steps-per-call rate and the host-state e2e step --
+    run at two ranks too, with the same collectives on every rank, and rank 0
+    prints one line that carries them all."""
+    port = _free_port()
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py", "--gpus", "2",
+           "--workload", "chain16_d9231114_dirichlet", "--steps", "2", "--warmup", "3",
+           "--no-cpu-baseline", "--e2e-steps", "1", "--fused-steps", "8"]
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES=os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0],
+               OMP_NUM_THREADS="1")
+    out = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=1500, env=env)
+    assert out.returncode == 0, out.stderr[-3000:]
+    lines = [json.loads(s) for s in out.stdout.splitlines() if s.startswith("{")]
+    assert len(lines) == 1, out.stdout[-2000:]
+    line = lines[0]
+    assert line["n_gpus"] == 2 and line["value"] > 0
+    names = [p["workload"] for p in line["per_workload"]]
+    assert "chain16_d9231114_dirichlet" not in names and len(names) >= 5, names
+    for p in line["per_workload"]:
+        assert p["value"] > 0 and p["roofline"]["frac"] > 0 and p["gpu_launches"] > 0, p
+    f = line["fused_steps"]
+    assert f["value"] > 0 and f["steps_per_call"] == 8
+    e = line["e2e"]
+    assert (e.get("value") or 0) > 0 or "skipped" in e, e
