@@ -69,3 +69,18 @@ def test_warmup_below_three_is_refused():
 
 if __name__ == "__main__":
     sys.exit(pytest.main([__file__, "-q"]))
+
+
+def test_traffic_entries_cover_the_default_line():
+    """Every workload of the default bench line (the headline and its
+    per-workload entries, all on the walk with stored centres) has a committed
+    ncu DRAM-traffic figure, so the line's roofline.traffic is never null
+    for a missing entry; the figures are of the order of the algorithmic bytes."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2110_04175_gb300 import workloads as wl
+    for name in [bench.DEFAULT_WORKLOAD] + bench.PER_WORKLOAD:
+        w = wl.by_name(name)
+        t = bench.traffic_per_launch(w, "stored", "relay_models_kernel", "sgd")
+        assert t is not None, name
+        assert 0.8 < t / w.bytes_per_step() < 1.3, (name, t, w.bytes_per_step())
